@@ -1,0 +1,375 @@
+"""Benchmark of the kNN-LM step (search + top-r + Eq. 2 + Eq. 3) on GB300.
+
+Default workload (``decode``): bf16 keys d=4096, N=1,048,576 from a 256-centre
+Gaussian mixture, values Zipf(1.1) over 32000 tokens, B=4 queries, r=1024,
+mu=1/64, lambda=0.8.  A step is one ``nest_knn_step`` over one batch.
+
+Prints ONE JSON line (rank 0): queries/s over all ranks, the scan kernel's
+HBM roofline fraction (CUDA events around that kernel, inside the timed
+region), the oracle timed on the host cores on a bounded sample, an
+end-to-end number through the public API with host buffers, and the SM
+clocks sampled during the timed region.
+
+``--impl reference`` times the fp64 CPU oracle instead (the only reference
+implementation this method has here), on a bounded sample of the same
+workload per step.
+
+Multi-GPU: each rank runs an independent decoding stream (its own datastore
+replica and query batches); nothing is exchanged, so ``scaling`` is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="decode", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--B", type=int, default=None, help="override the query batch")
+    p.add_argument("--N", type=int, default=None,
+                   help="override the datastore size (small cases for profiling)")
+    p.add_argument("--oracle-queries", type=int, default=2,
+                   help="queries in the oracle's bounded sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=200)
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(device_index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64,
+                     device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def host_keys(K: torch.Tensor, rows: int | None = None):
+    """Exact bytes of the first ``rows`` keys on the host (bf16 as uint16), ~1 GiB pieces."""
+    import numpy as np
+    n = K.shape[0] if rows is None else rows
+    step = max(1, (1 << 30) // (K.shape[1] * K.element_size()))
+    parts = []
+    for lo in range(0, n, step):
+        parts.append(synth.to_numpy_raw(K[lo:min(n, lo + step)]))
+    return np.concatenate(parts) if len(parts) > 1 else parts[0]
+
+
+class OracleSampler:
+    """Times the fp64 oracle, as it stands, on a bounded sample of the workload.
+
+    Full-scan workloads: ``nq`` queries against the first ``n`` keys (search,
+    top-r, Eq. 2, Eq. 3); the oracle's cost grows linearly with the keys
+    scanned, so queries/s over the whole datastore is (n / N) * nq / seconds.
+    Ragged workloads: ``nq`` queries, each over its own segment.
+    """
+
+    def __init__(self, w, x, nq: int, max_keys: int):
+        import oracle
+        oracle.build()
+        self.oracle = oracle
+        self.w, self.nq = w, nq
+        self.N = x.K.shape[0]
+        self.ragged = x.seg_off is not None
+        self.V = x.V.cpu().numpy()
+        self.q = synth.to_numpy_raw(x.q[:nq])
+        self.p_lm = x.p_lm[:nq].cpu().numpy()
+        if self.ragged:
+            so = x.seg_off[:nq + 1].cpu().numpy()
+            self.seg = so
+            self.K = host_keys(x.K, int(so[-1]))
+            self.n = int((so[1:] - so[:-1]).sum())
+        else:
+            self.K = host_keys(x.K, min(self.N, max_keys))
+            self.n = self.K.shape[0]
+        self.threads = oracle.default_threads()
+
+    def run(self, n: int | None = None) -> float:
+        """Seconds for one sample over the first n keys (all sampled keys by default)."""
+        w = self.w
+        t0 = time.perf_counter()
+        if self.ragged:
+            self.oracle.knn_step(self.K, self.V, self.q, w.r, self.p_lm, w.mu, w.lam, w.vocab,
+                                 seg_off=self.seg, nthreads=self.threads)
+        else:
+            n = self.n if n is None else n
+            self.oracle.knn_step(self.K[:n], self.V[:n], self.q, w.r, self.p_lm, w.mu, w.lam,
+                                 w.vocab, nthreads=self.threads)
+        return time.perf_counter() - t0
+
+    def fit(self, budget_s: float) -> int:
+        """Largest key count (from a short calibration) whose sample fits the budget."""
+        if self.ragged:
+            return self.n
+        probe = min(self.n, 16384)
+        t = self.run(probe)
+        n = int(probe * budget_s / max(t, 1e-6))
+        return max(min(self.n, n), min(self.n, 1024))
+
+    def queries_per_s(self, n: int, seconds: float) -> float:
+        if self.ragged:
+            return self.nq / seconds
+        return self.nq * (n / self.N) / seconds
+
+    def describe(self, n: int) -> str:
+        w = self.w
+        if self.ragged:
+            return (f"{self.nq} queries, each over its own candidate segment ({self.n} key "
+                    f"scans in all), top-{w.r}, Eq. 2 + Eq. 3 over {w.vocab} tokens")
+        return (f"{self.nq} queries against the first {n} of {self.N} keys, top-{w.r}, Eq. 2 + "
+                f"Eq. 3 over {w.vocab} tokens; queries/s scaled by {n}/{self.N} (cost is "
+                f"linear in the keys scanned)")
+
+
+def cpu_baseline(w, x, nq: int, budget_s: float = 15.0):
+    """The oracle on the host cores: one bounded sample of ~budget_s seconds."""
+    smp = OracleSampler(w, x, nq, max_keys=x.K.shape[0])
+    n = smp.fit(budget_s)
+    sec = smp.run(n)
+    return {"value": smp.queries_per_s(n, sec), "unit": "queries/s", "cores": smp.threads,
+            "kind": "oracle", "sample": smp.describe(n), "seconds": sec}
+
+
+def run_reference(args, w, world, rank):
+    """``--impl reference``: the oracle on the host cores, each step a bounded sample."""
+    if rank != 0:
+        return
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    x = synth.make_inputs(w, device=dev, B=args.B, N=args.N)
+    nq = min(args.oracle_queries, x.q.shape[0])
+    total_steps = args.steps + args.warmup
+    per_step = max(0.05, min(10.0, 150.0 / max(1, total_steps)))
+    smp = OracleSampler(w, x, nq, max_keys=x.K.shape[0])
+    n = smp.fit(per_step)
+    times = []
+    for i in range(total_steps):
+        t = smp.run(n)
+        if i >= args.warmup:
+            times.append(t)
+    total = sum(times)
+    value = smp.queries_per_s(n, total / len(times))
+    line = {
+        "impl": "reference", "metric": "queries/s for fused kNN search+top-r+p_M mix",
+        "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(w, x),
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": smp.threads,
+                         "kind": "oracle", "sample": smp.describe(n)},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_of(w, x):
+    B = x.q.shape[0]
+    return {"workload": w.name, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
+            "vocab": w.vocab, "key_dtype": w.dtype, "accumulate": "f32",
+            "mu": w.mu, "lambda": w.lam,
+            "ragged": bool(w.ragged),
+            "l2": "no flush: the keys streamed every step exceed the 129 MB L2"}
+
+
+def main():
+    args = parse()
+    w = synth.WORKLOADS[args.workload]
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, w, world, rank)
+        return
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU for the CUDA path")
+    torch.cuda.set_device(local)
+    import paper_2405_19325_gb300 as nest
+    from paper_2405_19325_gb300 import build as nest_build
+    nest_build.build()
+
+    dev = torch.device("cuda", local)
+    x = synth.make_inputs(w, device=dev, B=args.B, N=args.N, seed=w.seed + rank)
+    B = x.q.shape[0]
+    ds = nest.Datastore(x.K, x.V, w.vocab)
+    out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off)  # allocates scratch once
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off, out=out)
+    torch.cuda.synchronize()
+    if ds.device_status() != 0:
+        raise SystemExit("device status error during warm-up")
+
+    # ---- timed region: K steps, CUDA events on the launching stream
+    ds.timing_enable(True)
+    ds.timing_read()
+    launches0 = ds.launch_count()
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks = Clocks(local)
+    time.sleep(0.3)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off, out=out)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    ms_local = t0.elapsed_time(t1)
+    launches = ds.launch_count() - launches0
+    scan_ms, scan_n = ds.timing_read()
+    ds.timing_enable(False)
+    if ds.device_status() != 0:
+        raise SystemExit("device status error during the timed steps")
+    ms = max_over_ranks(ms_local, world)
+    value = world * B * args.steps / (ms / 1e3)
+
+    # ---- roofline of the dominant kernel (the key scan)
+    esize = 2 if w.dtype == "bf16" else 4
+    if x.seg_off is not None:
+        keys_scanned = int((x.seg_off[1:] - x.seg_off[:-1]).sum().item())
+    else:
+        keys_scanned = x.K.shape[0]
+    alg_bytes = keys_scanned * (w.d * esize + 4) + B * w.d * esize
+    scan_avg_ms = scan_ms / max(1, scan_n)
+    hbm_peak, peak_kind = peaks()
+    achieved = alg_bytes / (scan_avg_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": achieved / hbm_peak, "traffic": None, "kernel": "scan_topr_kernel",
+                "peak_kind": peak_kind, "alg_bytes_per_launch": alg_bytes,
+                "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
+
+    # ---- end to end through the public API with pinned host buffers
+    q_h = x.q.cpu().pin_memory()
+    p_h = x.p_lm.cpu().pin_memory()
+    so_h = x.seg_off.cpu().pin_memory() if x.seg_off is not None else None
+    staging = {}
+    for _ in range(3):
+        ds.step_host(q_h, w.r, p_h, w.mu, w.lam, seg_off_host=so_h, staging=staging)
+    barrier(world)
+    te = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        ds.step_host(q_h, w.r, p_h, w.mu, w.lam, seg_off_host=so_h, staging=staging)
+    e2e_s = max_over_ranks(time.perf_counter() - te, world)
+    h2d = q_h.numel() * q_h.element_size() + p_h.numel() * 4 + (
+        so_h.numel() * 8 if so_h is not None else 0)
+    d2h = B * w.vocab * 4 + B * w.r * 4 + B * w.r * 8
+    e2e = {"value": world * B * args.e2e_steps / e2e_s, "unit": "queries/s",
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, x, min(args.oracle_queries, B))
+        cpu.pop("seconds", None)
+
+    if rank == 0:
+        line = {
+            "metric": "queries/s for fused kNN search+top-r+p_M mix", "value": value,
+            "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
+            "data": "synthetic", "config": config_of(w, x),
+            "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    ds.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

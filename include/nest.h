@@ -1,0 +1,208 @@
+/*
+ * nest.h -- C ABI of the GB300 kNN-LM step of Nearest Neighbor Speculative
+ * Decoding (NEST, arXiv 2405.19325).
+ *
+ * One step of the method, for a batch of B LM hidden states q (the queries):
+ *
+ *   search  s(q, k) = -||q - k||^2 against every datastore key k, or, for the
+ *           second stage of NEST's two-stage search, against a per-query
+ *           candidate segment of the keys (Sec. 2.2; Sec. 3.1; App. A), and
+ *           keep the r nearest neighbours pi (Sec. 2.2; search step of
+ *           Algorithm 1);
+ *   mix     p_kNN(w) proportional to sum over pi of 1[w = v_i] exp(mu s_i)
+ *           (Eq. 2), then p_M = lambda p_LM + (1 - lambda) p_kNN (Eq. 3), or
+ *           with lambda replaced by the relative retrieval confidence
+ *           lambda_t of Eq. 4.
+ *
+ * Conventions shared by every call:
+ *   - Array arguments are DEVICE pointers on the current CUDA device, owned
+ *     by the caller, unless a comment says otherwise.  Matrices are dense and
+ *     row-major.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  All work is stream-ordered and no call synchronizes the
+ *     stream, except nest_datastore_create, nest_device_status and
+ *     nest_timing_read, which say so.
+ *   - Keys and queries are NEST_F32 or NEST_BF16 (IEEE bfloat16 bits).
+ *     Distances, similarities and probabilities are fp32.
+ *   - Argument errors are found on the host before anything is launched and
+ *     are returned synchronously.  Conditions only the GPU can see (a bad
+ *     segment offset, an out-of-range neighbour index, a wait that ran out
+ *     of time) are recorded in a per-datastore device status word and
+ *     reported by nest_device_status.
+ *   - A datastore handle is not safe for concurrent calls from several
+ *     streams or threads: its scratch memory is shared by its calls.
+ */
+#ifndef NEST_H
+#define NEST_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define NEST_API __attribute__((visibility("default")))
+#else
+#define NEST_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum nest_status {
+    NEST_OK = 0,
+    NEST_ERR_INVALID_ARG = 1,  /* null pointer, size out of range, bad lambda/tau */
+    NEST_ERR_DTYPE = 2,        /* unknown element type */
+    NEST_ERR_ALIGN = 3,        /* pointer or row not 16-byte aligned */
+    NEST_ERR_OOM = 4,          /* device allocation failed */
+    NEST_ERR_CUDA = 5,         /* a CUDA runtime call failed */
+    NEST_ERR_VALUE_RANGE = 6,  /* token id outside [0, vocab) or key index outside [0, N) */
+    NEST_ERR_OVERFLOW = 7,     /* reserved: a bounded device buffer overflowed */
+    NEST_ERR_TIMEOUT = 8,      /* a device-side wait gave up */
+    NEST_ERR_UNSUPPORTED = 9   /* shape outside what the kernels handle */
+} nest_status_t;
+
+typedef enum nest_dtype { NEST_F32 = 0, NEST_BF16 = 1 } nest_dtype_t;
+
+/* Largest r accepted by the search. */
+#define NEST_MAX_R 4096
+/* Largest row of a key or query, in bytes (d * element size). */
+#define NEST_MAX_ROW_BYTES 16384
+
+typedef struct nest_datastore nest_datastore_t;
+
+/*
+ * Register a key-value datastore (K, V) (Sec. 2.2, Eq. 1: key k_i = hidden
+ * state f(c_i), value v_i = the next token w_i).
+ *
+ *   K      N x d keys, element type `dtype`; 16-byte aligned, and a row
+ *          (d * element size bytes) must be a multiple of 16 bytes and at
+ *          most NEST_MAX_ROW_BYTES.
+ *   V      N token ids (int32), each in [0, vocab).
+ *   N      number of keys, 1 <= N <= 2^32 - 2.
+ *   vocab  vocabulary size of p_LM / p_kNN / p_M, >= 1.
+ *   out    receives the handle.
+ *
+ * K and V are BORROWED: the caller keeps them alive and unchanged until
+ * nest_datastore_destroy.  The handle owns the fp32 key norms ||k_i||^2
+ * (computed here, N * 4 bytes), a device status word and the scratch memory
+ * of later calls.  This call synchronizes `stream`: it checks every value
+ * on the device and returns NEST_ERR_VALUE_RANGE if one is out of range.
+ */
+NEST_API nest_status_t nest_datastore_create(const void* K, const int32_t* V, int64_t N, int32_t d,
+                                    nest_dtype_t dtype, int32_t vocab, void* stream,
+                                    nest_datastore_t** out);
+
+/* Free everything the handle owns (synchronizes the device).  NULL is a no-op. */
+NEST_API nest_status_t nest_datastore_destroy(nest_datastore_t* ds);
+
+/*
+ * Allocate the handle's scratch memory for searches of up to max_B queries
+ * and r <= max_r, so that such searches allocate nothing (for instance
+ * before stream capture).  Without it the first search of a larger shape
+ * allocates.  Synchronizes the device when it allocates.
+ */
+NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_B, int32_t max_r,
+                                     int32_t ragged);
+
+/*
+ * r-nearest-neighbour search (Sec. 2.2; Sec. 3.1 second stage; App. A).
+ *
+ *   q        B x d queries, the datastore's element type, 16-byte aligned.
+ *   B        1 <= B <= 65535.
+ *   r        1 <= r <= NEST_MAX_R.
+ *   seg_off  NULL: every query scans all N keys.  Otherwise B + 1 int64
+ *            offsets: query b scans only keys [seg_off[b], seg_off[b+1])
+ *            (its on-the-fly datastore K', given as a segment of K).
+ *            Offsets must satisfy 0 <= seg_off[b] <= seg_off[b+1] <= N; a
+ *            violating segment is searched as empty and recorded as
+ *            NEST_ERR_INVALID_ARG in the device status.
+ *   s_out    B x r fp32: s = -||q - k||^2 of the neighbours, nearest first
+ *            (s descending, ties by smaller key index).
+ *   idx_out  B x r int64 global key indices of the neighbours.
+ *
+ * When a query has fewer than r candidate keys the tail of its row is
+ * padded with s = -inf and idx = -1.  Distances are evaluated as
+ * ||q||^2 + ||k||^2 - 2 q.k in fp32 and clamped at 0.
+ */
+NEST_API nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                              const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                              void* stream);
+
+/*
+ * Eq. 2 and Eq. 3 for each query row b < B:
+ *
+ *   p_kNN[b][w] = sum_{i : V[idx_in[b][i]] = w} exp(mu s_i) / sum_j exp(mu s_j)
+ *   p_M[b][w]   = lambda p_LM[b][w] + (1 - lambda) p_kNN[b][w]
+ *
+ *   s_in, idx_in  B x r neighbours as written by nest_knn_search (entries
+ *                 with idx < 0 or s = -inf carry no weight; an index >= N
+ *                 is recorded as NEST_ERR_VALUE_RANGE and skipped).
+ *   p_lm          B x vocab fp32.
+ *   mu            inverse temperature (the paper uses 1/sqrt(d)).
+ *   lambda        in [0, 1].
+ *   p_knn_out     B x vocab fp32, or NULL when not wanted.
+ *   p_m_out       B x vocab fp32.
+ *
+ * A row with no real neighbour gets p_kNN = 0 and p_M = p_LM (lambda is
+ * taken as 1).  The softmax subtracts the largest s first, which leaves the
+ * result unchanged in exact arithmetic.
+ */
+NEST_API nest_status_t nest_knn_mix(nest_datastore_t* ds, const float* s_in, const int64_t* idx_in,
+                           const float* p_lm, int32_t B, int32_t r, float mu, float lambda,
+                           float* p_knn_out, float* p_m_out, void* stream);
+
+/*
+ * As nest_knn_mix, with each row's lambda replaced by the relative
+ * retrieval confidence of Eq. 4 (Sec. 3.2):
+ *
+ *   lambda_t = sigmoid((min_i |s_i| / max_i |s_i| - alpha) / tau)
+ *
+ * over the row's real neighbours (Eq. 4 takes absolute values, which the
+ * restatement in Algorithm 1 drops; Eq. 4 is followed).  tau > 0.  A row
+ * with no real neighbour gets lambda_t = 1; a row whose neighbours all have
+ * s = 0 takes the ratio as 1.  lambda_out (B fp32, or NULL) receives
+ * lambda_t.
+ */
+NEST_API nest_status_t nest_knn_mix_rrc(nest_datastore_t* ds, const float* s_in, const int64_t* idx_in,
+                               const float* p_lm, int32_t B, int32_t r, float mu, float alpha,
+                               float tau, float* lambda_out, float* p_knn_out, float* p_m_out,
+                               void* stream);
+
+/*
+ * One kNN-LM step: nest_knn_search followed by nest_knn_mix on `stream`,
+ * with the same arguments and outputs (s_out and idx_out are required; they
+ * carry the neighbours from the search to the mix).
+ */
+NEST_API nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                            const int64_t* seg_off, const float* p_lm, float mu, float lambda,
+                            float* s_out, int64_t* idx_out, float* p_knn_out, float* p_m_out,
+                            void* stream);
+
+/*
+ * Synchronize `stream`, return the first condition the GPU recorded for
+ * this datastore since the previous call (NEST_OK if none), and clear it.
+ */
+NEST_API nest_status_t nest_device_status(nest_datastore_t* ds, void* stream);
+
+/*
+ * Kernel timing: while enabled, every search records a pair of CUDA events
+ * on its stream around its distance-scan kernel (the kernel that streams
+ * the keys).  nest_timing_read synchronizes those events and returns the
+ * summed milliseconds and the number of launches since the last read.
+ */
+NEST_API nest_status_t nest_timing_enable(nest_datastore_t* ds, int32_t on);
+NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, int64_t* launches);
+
+/* Kernels this handle has launched since it was created (all kinds). */
+NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
+
+/* Static text for a status code. */
+NEST_API const char* nest_status_string(nest_status_t status);
+
+/* ABI version: major * 10000 + minor * 100 + patch. */
+NEST_API int32_t nest_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NEST_H */

@@ -1,0 +1,456 @@
+// api.cu -- the C ABI of include/nest.h: argument validation, the datastore
+// handle, scratch memory, and the choice and launch of the kernels.
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+
+using namespace nest;
+
+struct nest_datastore {
+    const void* K = nullptr;
+    const int32_t* V = nullptr;
+    int64_t N = 0;
+    int32_t d = 0;
+    int dtype = 0;
+    int32_t vocab = 0;
+    int32_t row_bytes = 0;
+    int device = 0;
+    int num_sms = 1;
+    size_t smem_optin = 0;
+    float* knorm = nullptr;  // owned: ||k_i||^2, N floats
+    int* status = nullptr;   // owned: device status word
+    uint64_t* scratch = nullptr;  // owned: candidate lists of the search
+    size_t scratch_words = 0;
+    bool timing = false;
+    std::vector<cudaEvent_t> events;  // pairs (start, end)
+    size_t events_used = 0;
+    int64_t launches = 0;
+};
+
+namespace {
+
+constexpr int64_t kMaxKeys = 4294967294LL;  // key indices travel as 32 bits
+constexpr int32_t kMaxB = 65535;
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+nest_status_t from_cuda(cudaError_t e)
+{
+    if (e == cudaSuccess) return NEST_OK;
+    if (e == cudaErrorMemoryAllocation) return NEST_ERR_OOM;
+    return NEST_ERR_CUDA;
+}
+
+cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+
+int element_size(int dtype) { return dtype == NEST_BF16 ? 2 : 4; }
+
+// Search layout chosen for a call: the scan kernel's plan and the merge tree.
+struct SearchPlan {
+    ScanPlan scan;
+    size_t cand_words;   // scan output: groups * parts * nq * r
+    size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
+};
+
+// Parts per query group: whole waves over the SMs, each part >= 256 keys.
+int choose_parts(int groups, int64_t keys_per_group, int num_sms, bool ragged)
+{
+    const int64_t by_keys = std::max<int64_t>(1, keys_per_group / 256);
+    const int max_parts = (int)std::min<int64_t>(ragged ? 64 : 1024, by_keys);
+    int best = 1;
+    double best_cost = 1e30;
+    for (int p = 1; p <= max_parts; ++p) {
+        const int64_t items = (int64_t)groups * p;
+        const int64_t waves = (items + num_sms - 1) / num_sms;
+        const double cost = (double)waves / p + 2e-3 * p;
+        if (cost < best_cost - 1e-12) {
+            best_cost = cost;
+            best = p;
+        }
+    }
+    return best;
+}
+
+nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, SearchPlan* sp)
+{
+    const int chunks = ds->row_bytes / 16;
+    const int cpt = chunks <= 256 ? 1 : (chunks <= 512 ? 2 : 4);
+    int nq = ragged ? 1 : (B >= 3 ? 4 : B);
+    ScanPlan p{};
+    while (!scan_plan_smem(ds->dtype, nq, cpt, r, ds->row_bytes, ds->smem_optin, &p)) {
+        if (nq == 1) return NEST_ERR_UNSUPPORTED;
+        nq /= 2;
+    }
+    p.groups = ragged ? B : (B + nq - 1) / nq;
+    const int64_t keys_per_group = ragged ? (ds->N + B - 1) / B : ds->N;
+    p.parts = choose_parts(p.groups, keys_per_group, ds->num_sms, ragged);
+    sp->scan = p;
+    sp->cand_words = (size_t)p.groups * p.parts * p.nq * r;
+    const int per = merge_lists_per_cta(r);
+    const int lvl1 = (p.parts + per - 1) / per;
+    sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
+    return NEST_OK;
+}
+
+nest_status_t ensure_scratch(nest_datastore* ds, size_t words)
+{
+    if (words <= ds->scratch_words) return NEST_OK;
+    if (ds->scratch) {
+        cudaError_t e = cudaFree(ds->scratch);
+        ds->scratch = nullptr;
+        ds->scratch_words = 0;
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    void* p = nullptr;
+    cudaError_t e = cudaMalloc(&p, words * sizeof(uint64_t));
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return NEST_ERR_OOM;
+    }
+    ds->scratch = static_cast<uint64_t*>(p);
+    ds->scratch_words = words;
+    return NEST_OK;
+}
+
+nest_status_t record_event(nest_datastore* ds, cudaStream_t stream)
+{
+    if (ds->events_used == ds->events.size()) {
+        cudaEvent_t ev;
+        cudaError_t e = cudaEventCreate(&ev);
+        if (e != cudaSuccess) return from_cuda(e);
+        ds->events.push_back(ev);
+    }
+    return from_cuda(cudaEventRecord(ds->events[ds->events_used++], stream));
+}
+
+// Device pointers only: plain host memory would fault on GPUs that cannot reach it.
+bool is_device_pointer(const void* p)
+{
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+nest_status_t check_search_args(const nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                                const int64_t* seg_off, const float* s_out,
+                                const int64_t* idx_out)
+{
+    if (!ds || !q || !s_out || !idx_out) return NEST_ERR_INVALID_ARG;
+    if (B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R) return NEST_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(s_out, 4) || !aligned(idx_out, 8)) return NEST_ERR_ALIGN;
+    if (seg_off && !aligned(seg_off, 8)) return NEST_ERR_ALIGN;
+    return NEST_OK;
+}
+
+nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const int64_t* idx_in,
+                             const float* p_lm, int32_t B, int32_t r, const float* p_knn_out,
+                             const float* p_m_out)
+{
+    if (!ds || !s_in || !idx_in || !p_lm || !p_m_out) return NEST_ERR_INVALID_ARG;
+    if (B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R) return NEST_ERR_INVALID_ARG;
+    if (!aligned(s_in, 4) || !aligned(idx_in, 8) || !aligned(p_lm, 4) || !aligned(p_m_out, 4) ||
+        (p_knn_out && !aligned(p_knn_out, 4)))
+        return NEST_ERR_ALIGN;
+    return NEST_OK;
+}
+
+nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                         const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                         cudaStream_t stream)
+{
+    SearchPlan sp;
+    nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
+    if (st != NEST_OK) return st;
+    st = ensure_scratch(ds, sp.cand_words + sp.level_words);
+    if (st != NEST_OK) return st;
+
+    uint64_t* regionA = ds->scratch;
+    uint64_t* regionB = ds->scratch + sp.cand_words;
+
+    ScanArgs sa{};
+    sa.K = ds->K;
+    sa.knorm = ds->knorm;
+    sa.q = q;
+    sa.seg_off = seg_off;
+    sa.cand = regionA;
+    sa.status = ds->status;
+    sa.N = ds->N;
+    sa.row_bytes = ds->row_bytes;
+    sa.chunks = ds->row_bytes / 16;
+    sa.B = B;
+    sa.r = r;
+    sa.cap = sp.scan.cap;
+    sa.parts = sp.scan.parts;
+    sa.stages = sp.scan.stages;
+    sa.stage_bytes = sp.scan.stage_bytes;
+
+    if (ds->timing && (st = record_event(ds, stream)) != NEST_OK) return st;
+    cudaError_t e = launch_scan(ds->dtype, sp.scan, sa, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
+    if (ds->timing && (st = record_event(ds, stream)) != NEST_OK) return st;
+
+    MergeArgs ma{};
+    ma.in = regionA;
+    ma.list_stride = (int64_t)sp.scan.nq * r;
+    ma.nq_in = sp.scan.nq;
+    ma.lists = sp.scan.parts;
+    ma.B = B;
+    ma.r = r;
+    ma.s_out = s_out;
+    ma.idx_out = idx_out;
+    bool into_b = true;
+    for (;;) {
+        ma.per_cta = std::min(merge_lists_per_cta(r), ma.lists);
+        const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
+        const bool last = groups == 1;
+        ma.out = into_b ? regionB : regionA;
+        e = launch_merge(ma, last, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        ++ds->launches;
+        if (last) break;
+        ma.in = ma.out;
+        ma.list_stride = r;
+        ma.nq_in = 1;
+        ma.lists = groups;
+        into_b = !into_b;
+    }
+    return NEST_OK;
+}
+
+nest_status_t run_mix(nest_datastore* ds, const float* s_in, const int64_t* idx_in,
+                      const float* p_lm, int32_t B, int32_t r, float mu, float lambda, int rrc,
+                      float alpha, float tau, float* lam_out, float* p_knn_out, float* p_m_out,
+                      cudaStream_t stream)
+{
+    MixArgs m{};
+    m.s = s_in;
+    m.idx = idx_in;
+    m.V = ds->V;
+    m.p_lm = p_lm;
+    m.p_knn = p_knn_out;
+    m.p_m = p_m_out;
+    m.lam_out = lam_out;
+    m.status = ds->status;
+    m.N = ds->N;
+    m.vocab = ds->vocab;
+    m.B = B;
+    m.r = r;
+    m.mu = mu;
+    m.lambda = lambda;
+    m.rrc = rrc;
+    m.alpha = alpha;
+    m.tau = tau;
+    // Enough CTAs to stream the vocabulary rows, at least one per query.
+    const int64_t want = std::max<int64_t>(1, (2LL * ds->num_sms + B - 1) / B);
+    const int64_t by_vocab = std::max<int64_t>(1, ds->vocab / 2048);
+    m.slices = (int32_t)std::min<int64_t>(want, by_vocab);
+    cudaError_t e = launch_mix(m, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
+    return NEST_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+nest_status_t nest_datastore_create(const void* K, const int32_t* V, int64_t N, int32_t d,
+                                    nest_dtype_t dtype, int32_t vocab, void* stream,
+                                    nest_datastore_t** out)
+{
+    if (!out) return NEST_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!K || !V) return NEST_ERR_INVALID_ARG;
+    if (dtype != NEST_F32 && dtype != NEST_BF16) return NEST_ERR_DTYPE;
+    if (N < 1 || N > kMaxKeys || d < 1 || vocab < 1) return NEST_ERR_INVALID_ARG;
+    const int64_t row_bytes = (int64_t)d * element_size(dtype);
+    if (row_bytes > NEST_MAX_ROW_BYTES) return NEST_ERR_UNSUPPORTED;
+    if (row_bytes % 16 != 0 || !aligned(K, 16) || !aligned(V, 4)) return NEST_ERR_ALIGN;
+    if (!is_device_pointer(K) || !is_device_pointer(V)) return NEST_ERR_INVALID_ARG;
+
+    nest_datastore* ds = new (std::nothrow) nest_datastore();
+    if (!ds) return NEST_ERR_OOM;
+    ds->K = K;
+    ds->V = V;
+    ds->N = N;
+    ds->d = d;
+    ds->dtype = dtype;
+    ds->vocab = vocab;
+    ds->row_bytes = (int32_t)row_bytes;
+    cudaError_t e = cudaGetDevice(&ds->device);
+    int optin = 0;
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&ds->num_sms, cudaDevAttrMultiProcessorCount, ds->device);
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, ds->device);
+    ds->smem_optin = (size_t)optin;
+    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ds->knorm), (size_t)N * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ds->status), sizeof(int));
+    cudaStream_t st = as_stream(stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ds->status, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = launch_key_norms(K, N, d, dtype, ds->knorm, st);
+    if (e == cudaSuccess) e = launch_check_values(V, N, vocab, ds->status, st);
+    int host_status = 0;
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&host_status, ds->status, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        nest_datastore_destroy(ds);
+        return e == cudaErrorMemoryAllocation ? NEST_ERR_OOM : NEST_ERR_CUDA;
+    }
+    ds->launches = 2;
+    if (host_status != 0) {
+        nest_datastore_destroy(ds);
+        return static_cast<nest_status_t>(host_status);
+    }
+    *out = ds;
+    return NEST_OK;
+}
+
+nest_status_t nest_datastore_destroy(nest_datastore_t* ds)
+{
+    if (!ds) return NEST_OK;
+    cudaError_t first = cudaSuccess;
+    auto keep = [&](cudaError_t e) {
+        if (first == cudaSuccess) first = e;
+    };
+    if (ds->knorm) keep(cudaFree(ds->knorm));
+    if (ds->status) keep(cudaFree(ds->status));
+    if (ds->scratch) keep(cudaFree(ds->scratch));
+    for (cudaEvent_t ev : ds->events) keep(cudaEventDestroy(ev));
+    delete ds;
+    return from_cuda(first);
+}
+
+nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_B, int32_t max_r,
+                                     int32_t ragged)
+{
+    if (!ds || max_B < 1 || max_B > kMaxB || max_r < 1 || max_r > NEST_MAX_R)
+        return NEST_ERR_INVALID_ARG;
+    size_t need = 0;
+    for (int r = 1; r <= max_r; r = (r == max_r) ? max_r + 1 : std::min(max_r, r * 2)) {
+        for (int B = 1; B <= max_B; B = (B == max_B) ? max_B + 1 : std::min(max_B, B * 2)) {
+            SearchPlan sp;
+            if (plan_search(ds, B, r, ragged != 0, &sp) == NEST_OK)
+                need = std::max(need, sp.cand_words + sp.level_words);
+        }
+    }
+    return ensure_scratch(ds, need);
+}
+
+nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                              const int64_t* seg_off, float* s_out, int64_t* idx_out, void* stream)
+{
+    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st != NEST_OK) return st;
+    return run_search(ds, q, B, r, seg_off, s_out, idx_out, as_stream(stream));
+}
+
+nest_status_t nest_knn_mix(nest_datastore_t* ds, const float* s_in, const int64_t* idx_in,
+                           const float* p_lm, int32_t B, int32_t r, float mu, float lambda,
+                           float* p_knn_out, float* p_m_out, void* stream)
+{
+    nest_status_t st = check_mix_args(ds, s_in, idx_in, p_lm, B, r, p_knn_out, p_m_out);
+    if (st != NEST_OK) return st;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return NEST_ERR_INVALID_ARG;
+    return run_mix(ds, s_in, idx_in, p_lm, B, r, mu, lambda, 0, 0.f, 1.f, nullptr, p_knn_out,
+                   p_m_out, as_stream(stream));
+}
+
+nest_status_t nest_knn_mix_rrc(nest_datastore_t* ds, const float* s_in, const int64_t* idx_in,
+                               const float* p_lm, int32_t B, int32_t r, float mu, float alpha,
+                               float tau, float* lambda_out, float* p_knn_out, float* p_m_out,
+                               void* stream)
+{
+    nest_status_t st = check_mix_args(ds, s_in, idx_in, p_lm, B, r, p_knn_out, p_m_out);
+    if (st != NEST_OK) return st;
+    if (!(tau > 0.f) || alpha != alpha) return NEST_ERR_INVALID_ARG;
+    if (lambda_out && !aligned(lambda_out, 4)) return NEST_ERR_ALIGN;
+    return run_mix(ds, s_in, idx_in, p_lm, B, r, mu, 0.f, 1, alpha, tau, lambda_out, p_knn_out,
+                   p_m_out, as_stream(stream));
+}
+
+nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                            const int64_t* seg_off, const float* p_lm, float mu, float lambda,
+                            float* s_out, int64_t* idx_out, float* p_knn_out, float* p_m_out,
+                            void* stream)
+{
+    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st != NEST_OK) return st;
+    st = check_mix_args(ds, s_out, idx_out, p_lm, B, r, p_knn_out, p_m_out);
+    if (st != NEST_OK) return st;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return NEST_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    st = run_search(ds, q, B, r, seg_off, s_out, idx_out, s);
+    if (st != NEST_OK) return st;
+    return run_mix(ds, s_out, idx_out, p_lm, B, r, mu, lambda, 0, 0.f, 1.f, nullptr, p_knn_out,
+                   p_m_out, s);
+}
+
+nest_status_t nest_device_status(nest_datastore_t* ds, void* stream)
+{
+    if (!ds) return NEST_ERR_INVALID_ARG;
+    cudaStream_t st = as_stream(stream);
+    int h = 0;
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemcpy(&h, ds->status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemset(ds->status, 0, sizeof(int));
+    if (e != cudaSuccess) return from_cuda(e);
+    return static_cast<nest_status_t>(h);
+}
+
+nest_status_t nest_timing_enable(nest_datastore_t* ds, int32_t on)
+{
+    if (!ds) return NEST_ERR_INVALID_ARG;
+    ds->timing = on != 0;
+    return NEST_OK;
+}
+
+nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, int64_t* launches)
+{
+    if (!ds || !total_ms || !launches) return NEST_ERR_INVALID_ARG;
+    double sum = 0.0;
+    const size_t pairs = ds->events_used / 2;
+    for (size_t i = 0; i < pairs; ++i) {
+        cudaError_t e = cudaEventSynchronize(ds->events[2 * i + 1]);
+        float ms = 0.f;
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, ds->events[2 * i], ds->events[2 * i + 1]);
+        if (e != cudaSuccess) return from_cuda(e);
+        sum += ms;
+    }
+    *total_ms = sum;
+    *launches = (int64_t)pairs;
+    ds->events_used = 0;
+    return NEST_OK;
+}
+
+int64_t nest_launch_count(const nest_datastore_t* ds) { return ds ? ds->launches : 0; }
+
+const char* nest_status_string(nest_status_t s)
+{
+    switch (s) {
+    case NEST_OK: return "ok";
+    case NEST_ERR_INVALID_ARG: return "invalid argument";
+    case NEST_ERR_DTYPE: return "unknown element type";
+    case NEST_ERR_ALIGN: return "pointer or row not 16-byte aligned";
+    case NEST_ERR_OOM: return "device allocation failed";
+    case NEST_ERR_CUDA: return "CUDA runtime error";
+    case NEST_ERR_VALUE_RANGE: return "token id or key index out of range";
+    case NEST_ERR_OVERFLOW: return "device buffer overflow";
+    case NEST_ERR_TIMEOUT: return "device wait timed out";
+    case NEST_ERR_UNSUPPORTED: return "shape not supported";
+    }
+    return "unknown status";
+}
+
+int32_t nest_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,113 @@
+// internal.h -- declarations shared by the library's translation units
+// (host launchers of the kernels; constants of the candidate encoding).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/nest.h"
+
+namespace nest {
+
+// A candidate neighbour is one 64-bit word: the fp32 bits of its squared
+// distance (non-negative, so the bits order like the values) above its
+// 32-bit key index.  Ordering the words orders neighbours nearest first
+// with ties broken by the smaller key index.  kNoCandidate pads lists.
+constexpr uint64_t kNoCandidate = ~0ull;
+
+// Device status word: the first recorded nest_status_t value wins.
+__device__ __forceinline__ void record_status(int* status, int code)
+{
+    atomicCAS(status, 0, code);
+}
+
+// ---------------------------------------------------------------- norms.cu
+cudaError_t launch_key_norms(const void* K, int64_t N, int32_t d, int dtype, float* knorm,
+                             cudaStream_t stream);
+cudaError_t launch_check_values(const int32_t* V, int64_t N, int32_t vocab, int* status,
+                                cudaStream_t stream);
+
+// ---------------------------------------------------------------- scan.cu
+// Distance scan with fused per-CTA top-r (decode / ragged regime).
+struct ScanPlan {
+    int nq;           // queries per CTA (1, 2 or 4)
+    int cpt;          // 16-byte chunks of a row per consumer thread (1, 2 or 4)
+    int groups;       // query groups
+    int parts;        // key-range parts per group
+    int cap;          // candidate buffer entries per query
+    int stages;       // pipeline depth
+    int stage_bytes;  // bytes of one stage (kScanRows rows)
+    size_t smem;      // dynamic shared memory of one CTA
+};
+
+constexpr int kScanRows = 4;           // key rows per pipeline stage
+constexpr int kScanThreads = 288;      // 8 consumer warps + 1 producer warp
+
+struct ScanArgs {
+    const void* K;
+    const float* knorm;
+    const void* q;
+    const int64_t* seg_off;  // nullptr: full scan
+    uint64_t* cand;          // [groups * parts][nq][r] candidate lists
+    int* status;
+    int64_t N;
+    int32_t row_bytes;
+    int32_t chunks;  // 16-byte chunks per row
+    int32_t B;
+    int32_t r;
+    int32_t cap;
+    int32_t parts;
+    int32_t stages;
+    int32_t stage_bytes;
+};
+
+// Returns false if no kernel exists for (dtype, nq, cpt).
+bool scan_plan_smem(int dtype, int nq, int cpt, int r, int row_bytes, size_t smem_limit,
+                    ScanPlan* plan);
+cudaError_t launch_scan(int dtype, const ScanPlan& plan, const ScanArgs& args,
+                        cudaStream_t stream);
+
+// ---------------------------------------------------------------- merge.cu
+// Merge candidate lists of each query into its top r.
+struct MergeArgs {
+    const uint64_t* in;    // candidate lists
+    int64_t list_stride;   // entries between consecutive lists of one query
+    int32_t nq_in;         // query b's first list is at ((b / nq_in) * lists * nq_in + b % nq_in) * r
+    int32_t lists;         // lists per query
+    int32_t per_cta;       // lists merged by one CTA
+    int32_t B;
+    int32_t r;
+    uint64_t* out;         // next level: [B][ceil(lists / per_cta)][r]; unused on the last level
+    float* s_out;          // last level only: B x r
+    int64_t* idx_out;      // last level only: B x r
+};
+
+int merge_lists_per_cta(int r);
+size_t merge_smem_bytes(int per_cta, int r);
+cudaError_t launch_merge(const MergeArgs& args, bool last, cudaStream_t stream);
+
+// ---------------------------------------------------------------- mix.cu
+struct MixArgs {
+    const float* s;
+    const int64_t* idx;
+    const int32_t* V;
+    const float* p_lm;
+    float* p_knn;    // may be null
+    float* p_m;
+    float* lam_out;  // may be null
+    int* status;
+    int64_t N;
+    int32_t vocab;
+    int32_t B;
+    int32_t r;
+    float mu;
+    float lambda;
+    int32_t rrc;  // 1: Eq. 4 lambda_t from (alpha, tau)
+    float alpha;
+    float tau;
+    int32_t slices;  // vocabulary slices per query (grid.x)
+};
+
+cudaError_t launch_mix(const MixArgs& args, cudaStream_t stream);
+
+}  // namespace nest

@@ -1,0 +1,158 @@
+// merge.cu -- combine per-CTA candidate lists into each query's r nearest
+// neighbours (the selection of pi, Sec. 2.2 / Algorithm 1's search step).
+//
+// A CTA loads up to per_cta lists of one query into shared memory (dropping
+// empty slots), keeps the r smallest words with the same radix select the
+// scan uses, and either writes them as one list for the next level or, on
+// the last level, sorts them (bitonic) and writes s = -distance and the key
+// index, nearest first, ties by smaller index, padding with (-inf, -1).
+#include <cmath>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "select.cuh"
+
+namespace nest {
+namespace {
+
+constexpr int kMergeThreads = 1024;
+constexpr size_t kMergeBufBytes = 192 * 1024;
+
+struct MergeShared {
+    uint64_t thr;
+    int cnt;
+    int wcnt[2][kMergeThreads / 32];
+    SelectSmem<kMergeThreads, 1> sel;
+};
+
+__host__ __device__ inline int next_pow2(int x)
+{
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+__host__ __device__ inline size_t buf_words(int per_cta, int r)
+{
+    const size_t a = (size_t)per_cta * r, b = (size_t)next_pow2(r);
+    return a > b ? a : b;
+}
+
+template <bool LAST>
+__global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs a)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint64_t* buf = reinterpret_cast<uint64_t*>(smem);
+    MergeShared& sh = *reinterpret_cast<MergeShared*>(smem + buf_words(a.per_cta, a.r) * 8);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int b = blockIdx.y, grp = blockIdx.x;
+    const int l0 = grp * a.per_cta;
+    const int l1 = min(a.lists, l0 + a.per_cta);
+    const uint64_t* src =
+        a.in + ((int64_t)(b / a.nq_in) * a.lists * a.nq_in + b % a.nq_in) * (int64_t)a.r;
+
+    // Load the lists, keeping real candidates only, in list order.
+    const int total = (l1 - l0) * a.r;
+    int n = 0;
+    for (int base = 0, t = 0; base < total; base += kMergeThreads, ++t) {
+        const int j = base + tid;
+        uint64_t e = kNoCandidate;
+        if (j < total) {
+            const int l = l0 + j / a.r, k = j - (j / a.r) * a.r;
+            e = src[(int64_t)l * a.list_stride + k];
+        }
+        const bool keep = e != kNoCandidate;
+        const uint32_t bal = __ballot_sync(~0u, keep);
+        if (lane == 0) sh.wcnt[t & 1][warp] = __popc(bal);
+        __syncthreads();
+        int before = 0, tot = 0;
+#pragma unroll
+        for (int w = 0; w < kMergeThreads / 32; ++w) {
+            const int c = sh.wcnt[t & 1][w];
+            before += (w < warp) ? c : 0;
+            tot += c;
+        }
+        if (keep) buf[n + before + __popc(bal & lanemask_lt())] = e;
+        n += tot;
+    }
+    if (tid == 0) {
+        sh.cnt = n;
+        sh.thr = kNoCandidate;
+    }
+    __syncthreads();
+    select_smallest<kMergeThreads, 1>(buf, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
+                                      [] { __syncthreads(); });
+    n = sh.cnt;
+
+    if constexpr (!LAST) {
+        uint64_t* dst = a.out + ((int64_t)b * gridDim.x + grp) * a.r;
+        for (int j = tid; j < a.r; j += kMergeThreads) dst[j] = j < n ? buf[j] : kNoCandidate;
+    } else {
+        const int P2 = next_pow2(n > 0 ? n : 1);
+        for (int j = n + tid; j < P2; j += kMergeThreads) buf[j] = kNoCandidate;
+        __syncthreads();
+        for (int k = 2; k <= P2; k <<= 1) {
+            for (int jj = k >> 1; jj > 0; jj >>= 1) {
+                for (int i = tid; i < P2; i += kMergeThreads) {
+                    const int l = i ^ jj;
+                    if (l > i) {
+                        const uint64_t x = buf[i], y = buf[l];
+                        const bool ascending = (i & k) == 0;
+                        if ((x > y) == ascending) {
+                            buf[i] = y;
+                            buf[l] = x;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        float* so = a.s_out + (int64_t)b * a.r;
+        int64_t* io = a.idx_out + (int64_t)b * a.r;
+        for (int j = tid; j < a.r; j += kMergeThreads) {
+            if (j < n) {
+                const uint64_t e = buf[j];
+                so[j] = -__uint_as_float((uint32_t)(e >> 32));
+                io[j] = (int64_t)(uint32_t)e;
+            } else {
+                so[j] = -INFINITY;
+                io[j] = -1;
+            }
+        }
+    }
+}
+
+}  // namespace
+
+int merge_lists_per_cta(int r)
+{
+    const int per = (int)(kMergeBufBytes / ((size_t)r * 8));
+    return per < 2 ? 2 : per;
+}
+
+size_t merge_smem_bytes(int per_cta, int r)
+{
+    return buf_words(per_cta, r) * 8 + sizeof(MergeShared);
+}
+
+cudaError_t launch_merge(const MergeArgs& a, bool last, cudaStream_t stream)
+{
+    const int groups = (a.lists + a.per_cta - 1) / a.per_cta;
+    const size_t smem = merge_smem_bytes(a.per_cta, a.r);
+    const dim3 grid(groups, a.B);
+    cudaError_t e;
+    if (last) {
+        e = cudaFuncSetAttribute(merge_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+        if (e != cudaSuccess) return e;
+        merge_kernel<true><<<grid, kMergeThreads, smem, stream>>>(a);
+    } else {
+        e = cudaFuncSetAttribute(merge_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+        if (e != cudaSuccess) return e;
+        merge_kernel<false><<<grid, kMergeThreads, smem, stream>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace nest

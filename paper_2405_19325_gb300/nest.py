@@ -1,0 +1,284 @@
+"""ctypes binding of the C ABI in include/nest.h (argument marshalling only).
+
+Every step of the kNN-LM path runs in the CUDA kernels of ``libnest.so``;
+this module only checks tensor properties, passes device pointers and the
+current torch stream, and raises on a non-zero status.  There is no CPU
+fallback: if the library is missing or no GPU is present, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libnest.so")
+
+F32 = 0
+BF16 = 1
+
+STATUS = {
+    0: "NEST_OK", 1: "NEST_ERR_INVALID_ARG", 2: "NEST_ERR_DTYPE", 3: "NEST_ERR_ALIGN",
+    4: "NEST_ERR_OOM", 5: "NEST_ERR_CUDA", 6: "NEST_ERR_VALUE_RANGE", 7: "NEST_ERR_OVERFLOW",
+    8: "NEST_ERR_TIMEOUT", 9: "NEST_ERR_UNSUPPORTED",
+}
+STATUS_CODE = {v: k for k, v in STATUS.items()}
+
+# Every entry point of include/nest.h: (name, restype, argtypes).
+_P = ctypes.c_void_p
+_I32, _I64, _F = ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+SIGNATURES = {
+    "nest_datastore_create": (ctypes.c_int, [_P, _P, _I64, _I32, ctypes.c_int, _I32, _P,
+                                             ctypes.POINTER(_P)]),
+    "nest_datastore_destroy": (ctypes.c_int, [_P]),
+    "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
+    "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
+    "nest_knn_mix": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _P, _P, _P]),
+    "nest_knn_mix_rrc": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _F, _P, _P, _P, _P]),
+    "nest_knn_step": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _F, _F, _P, _P, _P, _P, _P]),
+    "nest_device_status": (ctypes.c_int, [_P, _P]),
+    "nest_timing_enable": (ctypes.c_int, [_P, _I32]),
+    "nest_timing_read": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_double),
+                                        ctypes.POINTER(_I64)]),
+    "nest_launch_count": (_I64, [_P]),
+    "nest_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "nest_version": (_I32, []),
+}
+
+_lib = None
+
+
+class NestError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        self.name = STATUS.get(code, f"status {code}")
+        super().__init__(f"{where}: {self.name}")
+
+
+def load_library(path: str | None = None):
+    """Load libnest.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"{p} is missing: build it with paper_2405_19325_gb300.build.build()")
+    lib = ctypes.CDLL(p)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(code: int, where: str) -> None:
+    if code != 0:
+        raise NestError(code, where)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"keys/queries must be float32 or bfloat16, got {t.dtype}")
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class Datastore:
+    """A key-value datastore (K, V) registered with the CUDA library (Eq. 1)."""
+
+    def __init__(self, K: torch.Tensor, V: torch.Tensor, vocab: int, stream=None):
+        lib = load_library()
+        if K.dim() != 2:
+            raise ValueError("K must be N x d")
+        self.N, self.d = K.shape
+        self.dtype = K.dtype
+        self.vocab = int(vocab)
+        if V.shape != (self.N,):
+            raise ValueError("V must hold one token id per key")
+        kp = _dev(K, "K")
+        vp = _dev(V, "V", torch.int32)
+        self._K, self._V = K, V  # borrowed by the library: keep them alive
+        h = ctypes.c_void_p()
+        _check(lib.nest_datastore_create(kp, vp, self.N, self.d, _dtype_code(K), self.vocab,
+                                         _stream(stream), ctypes.byref(h)),
+               "nest_datastore_create")
+        self._h = h
+        self._lib = lib
+
+    @property
+    def handle(self) -> int:
+        return self._h.value
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None and self._h.value:
+            self._lib.nest_datastore_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def reserve(self, max_B: int, max_r: int, ragged: bool = False) -> None:
+        _check(self._lib.nest_datastore_reserve(self._h, max_B, max_r, int(ragged)),
+               "nest_datastore_reserve")
+
+    # ------------------------------------------------------------ search / mix / step
+    def search(self, q: torch.Tensor, r: int, seg_off: torch.Tensor | None = None,
+               s_out: torch.Tensor | None = None, idx_out: torch.Tensor | None = None,
+               stream=None):
+        """r nearest neighbours of each query: (s [B, r] fp32, idx [B, r] int64)."""
+        B = q.shape[0]
+        if q.dtype != self.dtype or q.dim() != 2 or q.shape[1] != self.d:
+            raise ValueError("q must be B x d with the datastore's dtype")
+        s_out = torch.empty(B, r, dtype=torch.float32, device=q.device) if s_out is None else s_out
+        idx_out = torch.empty(B, r, dtype=torch.int64, device=q.device) if idx_out is None else idx_out
+        sp = _dev(seg_off, "seg_off", torch.int64) if seg_off is not None else None
+        _check(self._lib.nest_knn_search(self._h, _dev(q, "q"), B, r, sp,
+                                         _dev(s_out, "s_out", torch.float32),
+                                         _dev(idx_out, "idx_out", torch.int64), _stream(stream)),
+               "nest_knn_search")
+        return s_out, idx_out
+
+    def mix(self, s: torch.Tensor, idx: torch.Tensor, p_lm: torch.Tensor, mu: float, lam: float,
+            want_p_knn: bool = False, p_m_out=None, p_knn_out=None, stream=None):
+        """Eq. 2 + Eq. 3: p_M (and p_kNN when asked)."""
+        B, r = s.shape
+        p_m_out = torch.empty_like(p_lm) if p_m_out is None else p_m_out
+        if want_p_knn and p_knn_out is None:
+            p_knn_out = torch.empty_like(p_lm)
+        self._check_rows(p_lm, B)
+        _check(self._lib.nest_knn_mix(self._h, _dev(s, "s", torch.float32),
+                                      _dev(idx, "idx", torch.int64),
+                                      _dev(p_lm, "p_lm", torch.float32), B, r, float(mu), float(lam),
+                                      _dev(p_knn_out, "p_knn_out", torch.float32)
+                                      if p_knn_out is not None else None,
+                                      _dev(p_m_out, "p_m_out", torch.float32), _stream(stream)),
+               "nest_knn_mix")
+        return (p_m_out, p_knn_out) if want_p_knn else p_m_out
+
+    def mix_rrc(self, s: torch.Tensor, idx: torch.Tensor, p_lm: torch.Tensor, mu: float,
+                alpha: float, tau: float, want_p_knn: bool = False, stream=None):
+        """Eq. 2 + Eq. 4: (p_M, lambda_t[B]) (+ p_kNN when asked)."""
+        B, r = s.shape
+        self._check_rows(p_lm, B)
+        p_m = torch.empty_like(p_lm)
+        lam = torch.empty(B, dtype=torch.float32, device=p_lm.device)
+        p_knn = torch.empty_like(p_lm) if want_p_knn else None
+        _check(self._lib.nest_knn_mix_rrc(self._h, _dev(s, "s", torch.float32),
+                                          _dev(idx, "idx", torch.int64),
+                                          _dev(p_lm, "p_lm", torch.float32), B, r, float(mu),
+                                          float(alpha), float(tau), lam.data_ptr(),
+                                          p_knn.data_ptr() if p_knn is not None else None,
+                                          p_m.data_ptr(), _stream(stream)),
+               "nest_knn_mix_rrc")
+        return (p_m, lam, p_knn) if want_p_knn else (p_m, lam)
+
+    def step(self, q: torch.Tensor, r: int, p_lm: torch.Tensor, mu: float, lam: float,
+             seg_off: torch.Tensor | None = None, want_p_knn: bool = False, out: dict | None = None,
+             stream=None) -> dict:
+        """One kNN-LM step (search + Eq. 2 + Eq. 3) in one C call."""
+        B = q.shape[0]
+        if q.dtype != self.dtype or q.dim() != 2 or q.shape[1] != self.d:
+            raise ValueError("q must be B x d with the datastore's dtype")
+        self._check_rows(p_lm, B)
+        o = out if out is not None else {}
+        dev = q.device
+        if "s" not in o:
+            o["s"] = torch.empty(B, r, dtype=torch.float32, device=dev)
+            o["idx"] = torch.empty(B, r, dtype=torch.int64, device=dev)
+            o["p_m"] = torch.empty(B, self.vocab, dtype=torch.float32, device=dev)
+            if want_p_knn:
+                o["p_knn"] = torch.empty(B, self.vocab, dtype=torch.float32, device=dev)
+        pk = o.get("p_knn")
+        sp = _dev(seg_off, "seg_off", torch.int64) if seg_off is not None else None
+        _check(self._lib.nest_knn_step(self._h, _dev(q, "q"), B, r, sp,
+                                       _dev(p_lm, "p_lm", torch.float32), float(mu), float(lam),
+                                       _dev(o["s"], "s_out", torch.float32),
+                                       _dev(o["idx"], "idx_out", torch.int64),
+                                       _dev(pk, "p_knn_out", torch.float32) if pk is not None else None,
+                                       _dev(o["p_m"], "p_m_out", torch.float32), _stream(stream)),
+               "nest_knn_step")
+        return o
+
+    def step_host(self, q_host: torch.Tensor, r: int, p_lm_host: torch.Tensor, mu: float,
+                  lam: float, seg_off_host: torch.Tensor | None = None, staging: dict | None = None,
+                  stream=None) -> dict:
+        """One step from host (pinned) inputs to host outputs, copies on the stream.
+
+        The query batch, p_LM and segment offsets go host -> device, the step
+        runs, and p_M, s and idx come back device -> host; the call returns
+        after the stream has finished.  ``staging`` caches device and pinned
+        buffers between calls.
+        """
+        st = staging if staging is not None else {}
+        s = stream if stream is not None else torch.cuda.current_stream()
+        dev = torch.device("cuda", torch.cuda.current_device())
+        B = q_host.shape[0]
+        if "q" not in st:
+            st["q"] = torch.empty(q_host.shape, dtype=q_host.dtype, device=dev)
+            st["p_lm"] = torch.empty(p_lm_host.shape, dtype=torch.float32, device=dev)
+            if seg_off_host is not None:
+                st["seg_off"] = torch.empty(B + 1, dtype=torch.int64, device=dev)
+            st["host_p_m"] = torch.empty(B, self.vocab, dtype=torch.float32).pin_memory()
+            st["host_s"] = torch.empty(B, r, dtype=torch.float32).pin_memory()
+            st["host_idx"] = torch.empty(B, r, dtype=torch.int64).pin_memory()
+            st["out"] = {}
+        with torch.cuda.stream(s):
+            st["q"].copy_(q_host, non_blocking=True)
+            st["p_lm"].copy_(p_lm_host, non_blocking=True)
+            so = None
+            if seg_off_host is not None:
+                st["seg_off"].copy_(seg_off_host, non_blocking=True)
+                so = st["seg_off"]
+            o = self.step(st["q"], r, st["p_lm"], mu, lam, seg_off=so, out=st["out"], stream=s)
+            st["host_p_m"].copy_(o["p_m"], non_blocking=True)
+            st["host_s"].copy_(o["s"], non_blocking=True)
+            st["host_idx"].copy_(o["idx"], non_blocking=True)
+        s.synchronize()
+        return {"p_m": st["host_p_m"], "s": st["host_s"], "idx": st["host_idx"]}
+
+    # ------------------------------------------------------------ status / timing
+    def device_status(self, stream=None) -> int:
+        """Synchronize and return (and clear) the device status code."""
+        return int(self._lib.nest_device_status(self._h, _stream(stream)))
+
+    def check(self, stream=None) -> None:
+        _check(self.device_status(stream), "device status")
+
+    def timing_enable(self, on: bool = True) -> None:
+        _check(self._lib.nest_timing_enable(self._h, int(on)), "nest_timing_enable")
+
+    def timing_read(self) -> tuple[float, int]:
+        ms = ctypes.c_double()
+        n = ctypes.c_int64()
+        _check(self._lib.nest_timing_read(self._h, ctypes.byref(ms), ctypes.byref(n)),
+               "nest_timing_read")
+        return ms.value, n.value
+
+    def launch_count(self) -> int:
+        return int(self._lib.nest_launch_count(self._h))
+
+    def _check_rows(self, p_lm: torch.Tensor, B: int) -> None:
+        if p_lm.dim() != 2 or p_lm.shape[0] != B or p_lm.shape[1] != self.vocab:
+            raise ValueError(f"p_lm must be {B} x {self.vocab}")

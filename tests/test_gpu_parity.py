@@ -1,0 +1,291 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Seeded synthetic inputs shaped like the paper's workloads (tiny fp32 case,
+decode-batch full scan, ragged second-stage search) plus edge cases: ragged
+tails, d not a multiple of 64, B not a multiple of the query group, r > N,
+r = N, r = 1, empty and short segments, exact ties on integer lattices, a key
+equal to the query, the largest row and the largest r.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from parity import check_mix, check_mix_end_to_end, check_search
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def nest():
+    from paper_2405_19325_gb300 import build as nest_build
+    nest_build.build()
+    import paper_2405_19325_gb300 as pkg
+    pkg.load_library()
+    return pkg
+
+
+def _np(t):
+    return synth.to_numpy_raw(t)
+
+
+def _cand_counts(B, N, seg_off):
+    if seg_off is None:
+        return np.full(B, N)
+    so = seg_off.cpu().numpy()
+    return so[1:] - so[:-1]
+
+
+def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, exact=False,
+                  oracle_threads=None):
+    dev = torch.device("cuda")
+    K, V, q, p_lm = K.to(dev), V.to(dev), q.to(dev), p_lm.to(dev)
+    so = seg_off.to(dev) if seg_off is not None else None
+    ds = nest.Datastore(K, V, vocab)
+    out = ds.step(q, r, p_lm, mu, lam, seg_off=so, want_p_knn=True)
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    s_g = out["s"].cpu().numpy()
+    i_g = out["idx"].cpu().numpy()
+    K_np, q_np, V_np = _np(K), _np(q), V.cpu().numpy()
+    p_lm_np = p_lm.cpu().numpy()
+    so_np = seg_off.cpu().numpy() if seg_off is not None else None
+    ref = oracle.knn_step(K_np, V_np, q_np, r, p_lm_np, mu, lam, vocab, seg_off=so_np,
+                          nthreads=oracle_threads)
+    rows = check_search(s_g, i_g, ref["s"], ref["idx"], K_np, q_np, dtype,
+                        _cand_counts(q.shape[0], K.shape[0], seg_off), exact=exact)
+    check_mix(out["p_m"].cpu().numpy(), s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
+              p_knn_gpu=out["p_knn"].cpu().numpy())
+    check_mix_end_to_end(out["p_m"].cpu().numpy(), ref["p_m"], rows)
+    ds.close()
+    return out, ref, rows
+
+
+# ---------------------------------------------------------------- the paper-shaped workloads
+
+def test_tiny_workload(nest):
+    w = synth.WORKLOADS["tiny"]
+    x = synth.make_inputs(w)
+    _, _, rows = run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype)
+    assert len(rows) == w.B
+
+
+def test_decode_workload_full_size(nest):
+    """bf16 d=4096, N=1,048,576 clustered keys, B=4, r=1024: the benchmarked launch."""
+    w = synth.WORKLOADS["decode"]
+    x = synth.make_inputs(w, device="cuda")
+    run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype)
+
+
+def test_ragged_workload_full_size(nest):
+    """32 queries x 40 passages x 256 keys, segment offsets, r=64."""
+    w = synth.WORKLOADS["ragged"]
+    x = synth.make_inputs(w, device="cuda")
+    _, _, rows = run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
+                               seg_off=x.seg_off)
+    assert len(rows) >= w.B // 2
+
+
+# ---------------------------------------------------------------- shapes and edges
+
+def _random_case(N, d, B, vocab, dtype, seed, centres=8):
+    g = torch.Generator().manual_seed(seed)
+    c = torch.randn(centres, d, generator=g)
+    K = (c[torch.randint(0, centres, (N,), generator=g)] + 0.3 * torch.randn(N, d, generator=g))
+    q = (c[torch.randint(0, centres, (B,), generator=g)] + 0.3 * torch.randn(B, d, generator=g))
+    dt = synth.torch_dtype(dtype)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g) * 2, dim=1)
+    return K.to(dt), V, q.to(dt), p_lm
+
+
+@pytest.mark.parametrize("N,d,B,r,dtype", [
+    (20003, 72, 5, 33, "bf16"),      # ragged tail, d % 64 != 0, B % 4 != 0
+    (4099, 8, 3, 7, "bf16"),         # smallest bf16 row (16 bytes)
+    (3001, 4096, 2, 100, "f32"),     # fp32 4096: four chunks per thread, two queries
+    (2500, 8192, 1, 64, "bf16"),     # largest row (16 KiB), one query
+    (5000, 256, 9, 1, "f32"),        # r = 1
+    (9000, 128, 4, 2048, "bf16"),    # r > 1024: fewer queries per CTA
+    (1500, 64, 1, 4096, "f32"),      # r = NEST_MAX_R > N: padded rows
+    (600, 16, 6, 600, "f32"),        # r = N
+    (12, 32, 4, 16, "f32"),          # r > N, N below one stage per CTA
+])
+def test_shapes(nest, N, d, B, r, dtype):
+    K, V, q, p_lm = _random_case(N, d, B, 500, dtype, seed=N + d)
+    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 500, dtype)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_integer_lattice_is_bit_exact_with_ties(nest, dtype):
+    """Small-integer keys: distances exact in fp32, many exact ties -> identical lists."""
+    g = torch.Generator().manual_seed(11)
+    N, d, B, r = 7000, 16, 6, 300
+    K = torch.randint(-3, 4, (N, d), generator=g).float()
+    q = torch.randint(-3, 4, (B, d), generator=g).float()
+    dt = synth.torch_dtype(dtype)
+    V = torch.randint(0, 50, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, 50, generator=g), dim=1)
+    run_and_check(nest, K.to(dt), V, q.to(dt), p_lm, r, 0.25, 0.6, 50, dtype, exact=True)
+
+
+def test_duplicate_keys_tie_break_by_index(nest):
+    g = torch.Generator().manual_seed(12)
+    base = torch.randn(50, 32, generator=g)
+    K = base.repeat(40, 1)  # every key appears 40 times
+    q = base[:4] + 0.01
+    V = torch.randint(0, 20, (K.shape[0],), generator=g, dtype=torch.int32)
+    p_lm = torch.full((4, 20), 1 / 20)
+    out, ref, _ = run_and_check(nest, K, V, q, p_lm, 100, 0.2, 0.5, 20, "f32")
+    # copies of the nearest key come first, in index order
+    i = out["idx"].cpu().numpy()
+    for b in range(4):
+        assert i[b, :40].tolist() == list(range(b, 2000, 50))
+
+
+def test_key_equal_to_query_is_first_with_distance_zero(nest):
+    g = torch.Generator().manual_seed(13)
+    K = torch.randn(10000, 128, generator=g).to(torch.bfloat16)
+    q = K[[17, 9999, 4242]].clone()
+    V = torch.randint(0, 100, (10000,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(3, 100, generator=g), dim=1)
+    out, _, _ = run_and_check(nest, K, V, q, p_lm, 10, 1 / np.sqrt(128), 0.8, 100, "bf16")
+    assert out["idx"][:, 0].cpu().tolist() == [17, 9999, 4242]
+
+
+def test_ragged_edges(nest):
+    """Empty segment, segments shorter than r, unequal lengths, one long segment."""
+    g = torch.Generator().manual_seed(14)
+    lens = [0, 5, 37, 300, 4000, 0, 64, 1]
+    N = sum(lens) + 10
+    K = torch.randn(N, 256, generator=g).to(torch.bfloat16)
+    B = len(lens)
+    q = torch.randn(B, 256, generator=g).to(torch.bfloat16)
+    off = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int64) + 3
+    V = torch.randint(0, 77, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, 77, generator=g), dim=1)
+    out, _, _ = run_and_check(nest, K, V, q, p_lm, 64, 1 / 16, 0.7, 77, "bf16", seg_off=off)
+    # an empty segment has no neighbours, so p_M = p_LM there
+    p_m = out["p_m"].cpu()
+    assert torch.equal(p_m[0], p_lm[0]) and torch.equal(p_m[5], p_lm[5])
+
+
+def test_mix_rrc_matches_eq4(nest):
+    w = synth.WORKLOADS["tiny"]
+    x = synth.make_inputs(w)
+    dev = torch.device("cuda")
+    ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
+    s, idx = ds.search(x.q.to(dev), w.r)
+    p_lm = x.p_lm.to(dev)
+    for alpha, tau in [(0.3, 0.1), (0.2, 0.1), (0.9, 0.5)]:
+        p_m, lam, p_knn = ds.mix_rrc(s, idx, p_lm, w.mu, alpha, tau, want_p_knn=True)
+        torch.cuda.synchronize()
+        s_np, i_np = s.cpu().numpy(), idx.cpu().numpy()
+        lam_or = oracle.rrc(s_np.astype(np.float64), i_np, alpha, tau)
+        np.testing.assert_allclose(lam.cpu().numpy(), lam_or, rtol=0, atol=1e-6)
+        check_mix(p_m.cpu().numpy(), s_np, i_np, x.V.numpy(), x.p_lm.numpy(), w.mu, None,
+                  w.vocab, p_knn_gpu=p_knn.cpu().numpy(), lam_gpu=lam.cpu().numpy())
+    assert ds.device_status() == 0
+    ds.close()
+
+
+def test_mix_lambda_one_and_zero(nest):
+    w = synth.WORKLOADS["tiny"]
+    x = synth.make_inputs(w)
+    dev = torch.device("cuda")
+    ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
+    s, idx = ds.search(x.q.to(dev), w.r)
+    p_lm = x.p_lm.to(dev)
+    p1, k1 = ds.mix(s, idx, p_lm, w.mu, 1.0, want_p_knn=True)
+    p0, k0 = ds.mix(s, idx, p_lm, w.mu, 0.0, want_p_knn=True)
+    assert torch.equal(p1, p_lm)
+    assert torch.equal(p0, k0) and torch.equal(k0, k1)
+    np.testing.assert_allclose(k0.double().sum(1).cpu().numpy(), 1.0, atol=1e-5)
+    ds.close()
+
+
+# ---------------------------------------------------------------- device-side errors
+
+def test_bad_segment_offsets_are_reported(nest):
+    dev = torch.device("cuda")
+    K = torch.randn(100, 16, device=dev)
+    V = torch.zeros(100, dtype=torch.int32, device=dev)
+    ds = nest.Datastore(K, V, 4)
+    q = torch.randn(2, 16, device=dev)
+    off = torch.tensor([0, 50, 40], dtype=torch.int64, device=dev)  # decreasing
+    s, idx = ds.search(q, 5, seg_off=off)
+    assert ds.device_status() == nest.nest.STATUS_CODE["NEST_ERR_INVALID_ARG"]
+    assert (idx[1] == -1).all()
+    assert ds.device_status() == 0  # cleared
+    ds.close()
+
+
+def test_out_of_range_neighbour_index_is_reported(nest):
+    dev = torch.device("cuda")
+    K = torch.randn(100, 16, device=dev)
+    V = torch.zeros(100, dtype=torch.int32, device=dev)
+    ds = nest.Datastore(K, V, 4)
+    s = torch.tensor([[-1.0, -2.0]], device=dev)
+    idx = torch.tensor([[3, 100]], dtype=torch.int64, device=dev)
+    p_lm = torch.full((1, 4), 0.25, device=dev)
+    p_m = ds.mix(s, idx, p_lm, 1.0, 0.5)
+    assert ds.device_status() == nest.nest.STATUS_CODE["NEST_ERR_VALUE_RANGE"]
+    # the bad neighbour carries no weight: token 0 gets all kNN mass
+    np.testing.assert_allclose(p_m.cpu().numpy(), [[0.625, 0.125, 0.125, 0.125]], atol=1e-7)
+    ds.close()
+
+
+def test_create_rejects_out_of_range_values(nest):
+    dev = torch.device("cuda")
+    K = torch.randn(64, 16, device=dev)
+    V = torch.arange(64, dtype=torch.int32, device=dev)
+    with pytest.raises(nest.NestError) as e:
+        nest.Datastore(K, V, 10)
+    assert e.value.name == "NEST_ERR_VALUE_RANGE"
+
+
+def test_host_validation_on_gpu(nest):
+    dev = torch.device("cuda")
+    K = torch.randn(64, 16, device=dev)
+    V = torch.zeros(64, dtype=torch.int32, device=dev)
+    ds = nest.Datastore(K, V, 10)
+    q = torch.randn(1, 16, device=dev)
+    with pytest.raises(nest.NestError) as e:
+        ds.search(q, 0)
+    assert e.value.name == "NEST_ERR_INVALID_ARG"
+    with pytest.raises(nest.NestError) as e:
+        ds.search(q, 5000)
+    assert e.value.name == "NEST_ERR_INVALID_ARG"
+    s, idx = ds.search(q, 3)
+    with pytest.raises(nest.NestError) as e:
+        ds.mix(s, idx, torch.full((1, 10), 0.1, device=dev), 1.0, 1.5)
+    assert e.value.name == "NEST_ERR_INVALID_ARG"
+    ds.close()
+
+
+def test_timing_and_launch_count(nest):
+    w = synth.WORKLOADS["tiny"]
+    x = synth.make_inputs(w)
+    dev = torch.device("cuda")
+    ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
+    q, p_lm = x.q.to(dev), x.p_lm.to(dev)
+    ds.timing_enable(True)
+    n0 = ds.launch_count()
+    for _ in range(3):
+        ds.step(q, w.r, p_lm, w.mu, w.lam)
+    ms, n = ds.timing_read()
+    assert n == 3 and ms > 0
+    assert ds.launch_count() - n0 >= 9  # scan + merge + mix per step
+    ds.close()
+
+
+def test_step_host_matches_device_step(nest):
+    w = synth.WORKLOADS["tiny"]
+    x = synth.make_inputs(w)
+    dev = torch.device("cuda")
+    ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
+    host = ds.step_host(x.q.pin_memory(), w.r, x.p_lm.pin_memory(), w.mu, w.lam)
+    o = ds.step(x.q.to(dev), w.r, x.p_lm.to(dev), w.mu, w.lam)
+    assert torch.equal(host["p_m"], o["p_m"].cpu())
+    assert torch.equal(host["idx"], o["idx"].cpu())
+    ds.close()
