@@ -56,18 +56,21 @@ struct SearchPlan {
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
 };
 
-// Parts per query group: whole waves over the SMs, each part >= 256 keys.
+// Parts per query group.  Time ~ waves * (work per part + fixed cost per part),
+// the fixed cost (prologue, final selection, one more list to merge) being
+// worth about 64 keys of streaming; parts hold at least 256 keys.
 int choose_parts(int groups, int64_t keys_per_group, int num_sms, bool ragged)
 {
     const int64_t by_keys = std::max<int64_t>(1, keys_per_group / 256);
-    const int max_parts = (int)std::min<int64_t>(ragged ? 64 : 1024, by_keys);
+    const int max_parts = (int)std::min<int64_t>(ragged ? 256 : 4096, by_keys);
+    const double fixed = 64.0 / (double)std::max<int64_t>(1, keys_per_group);
     int best = 1;
     double best_cost = 1e30;
     for (int p = 1; p <= max_parts; ++p) {
         const int64_t items = (int64_t)groups * p;
         const int64_t waves = (items + num_sms - 1) / num_sms;
-        const double cost = (double)waves / p + 2e-3 * p;
-        if (cost < best_cost - 1e-12) {
+        const double cost = (double)waves * (1.0 / p + fixed);
+        if (cost < best_cost * (1 - 1e-9)) {
             best_cost = cost;
             best = p;
         }

@@ -41,7 +41,7 @@ struct ScanPlan {
 };
 
 constexpr int kScanRows = 4;           // key rows per pipeline stage
-constexpr int kScanThreads = 288;      // 8 consumer warps + 1 producer warp
+constexpr int kScanThreads = 320;      // 8 consumer warps, 1 producer warp, 1 selector warp
 
 struct ScanArgs {
     const void* K;

@@ -3,17 +3,25 @@
 //
 // One CTA owns a group of up to NQ queries and a contiguous range of key
 // rows (a slice of the datastore, or a slice of one query's candidate
-// segment).  A producer warp streams the rows through a ring of shared-memory
-// stages with 1-D TMA bulk copies (mbarrier-tracked, L2 evict-first); eight
-// consumer warps hold the queries in registers and compute q.k in fp32 FMA,
-// each thread owning fixed 16-byte column chunks of every row.  Per stage of
-// kScanRows rows the partial dot products are reduced across the CTA, turned
-// into squared distances ||q||^2 + ||k||^2 - 2 q.k, and every candidate that
-// can still enter its query's r nearest is appended to a shared-memory list.
-// When a list fills up, a radix select trims every list back to r and
-// tightens the admission threshold.  At the end the CTA writes its r best
-// candidates per query; merge.cu combines the CTAs.  No distance ever goes
-// to global memory.
+// segment).  Three warp roles, decoupled by mbarrier rings:
+//
+//   producer warp   streams the rows into a ring of shared-memory stages of
+//                   kScanRows rows with 1-D TMA bulk copies (L2 evict-first);
+//   8 consumer warps hold the queries in registers (each thread owns fixed
+//                   16-byte column chunks of every row) and compute q.k with
+//                   packed fp32 FMA (two lanes of the sum per instruction);
+//                   per stage a warp reduce-scatter leaves one partial dot
+//                   product per (row, query) and warp in a ring of partials;
+//   selector warp   adds the 8 partials, forms ||q||^2 + ||k||^2 - 2 q.k,
+//                   appends every candidate that can still enter its
+//                   query's r nearest to a shared-memory list, and, when a
+//                   list fills up, trims it back to r with a radix select
+//                   (which also tightens the admission threshold).
+//
+// No block-wide barrier is taken per stage: the consumers only wait for
+// data and for free slots of the partial ring.  At the end the selector
+// writes the CTA's r best candidates per query; merge.cu combines the CTAs.
+// No distance ever goes to global memory.
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -25,8 +33,12 @@ namespace {
 
 constexpr int kConsumerWarps = 8;
 constexpr int kConsumers = kConsumerWarps * 32;
-constexpr int kBarConsumers = 1;  // hardware barrier id used by the consumer warps
+constexpr int kProducerWarp = kConsumerWarps;
+constexpr int kSelectorWarp = kConsumerWarps + 1;
+static_assert((kSelectorWarp + 1) * 32 == kScanThreads, "warp roles must fill the block");
+constexpr int kBarSetup = 1;      // consumers + selector, once (query norms)
 constexpr int kMaxStages = 8;
+constexpr int kPartialRing = 16;  // stages of partial sums in flight (a power of two)
 
 template <int DT>
 struct Elem;
@@ -39,22 +51,18 @@ struct Elem<NEST_BF16> {
     static constexpr int kPerChunk = 8;
 };
 
-// 16 bytes of a row -> fp32 values (bf16 -> fp32 is exact).
+// 16 bytes of a row -> fp32 pairs (element 2p, element 2p + 1); bf16 -> fp32 is exact.
 template <int DT>
-__device__ __forceinline__ void unpack_chunk(const uint4& v, float* x)
+__device__ __forceinline__ void unpack_pairs(const uint4& v, float2* x)
 {
     if constexpr (DT == NEST_BF16) {
         const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            x[2 * i] = __uint_as_float(w[i] << 16);
-            x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-        }
+        for (int i = 0; i < 4; ++i)
+            x[i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xffff0000u));
     } else {
-        x[0] = __uint_as_float(v.x);
-        x[1] = __uint_as_float(v.y);
-        x[2] = __uint_as_float(v.z);
-        x[3] = __uint_as_float(v.w);
+        x[0] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+        x[1] = make_float2(__uint_as_float(v.z), __uint_as_float(v.w));
     }
 }
 
@@ -62,13 +70,14 @@ template <int NQ>
 struct ScanShared {
     uint64_t full[kMaxStages];
     uint64_t empty[kMaxStages];
+    uint64_t pfull[kPartialRing];
+    uint64_t pempty[kPartialRing];
     uint64_t thr[NQ];
     int cnt[NQ];
-    float qnorm[NQ];
-    int need_select[2];
+    float qnorm_part[kConsumerWarps][NQ];
     int abort;
     int issued;
-    SelectSmem<kConsumers, NQ> sel;
+    SelectSmem<32, NQ> sel;
 };
 
 // Warp reduce-scatter of NV values: afterwards lane l holds the warp-wide
@@ -103,10 +112,23 @@ __device__ __forceinline__ uint32_t query_lanes(int qb)
     return m;
 }
 
+// Bounded wait that records a timeout and raises the CTA's abort flag; once
+// the flag is up every later wait returns at once so the CTA drains.
+__device__ __forceinline__ void wait_or_abort(uint64_t* bar, uint32_t parity, int* abort_flag,
+                                              int* status)
+{
+    if (*reinterpret_cast<volatile int*>(abort_flag)) return;
+    if (!mbar_wait_bounded(bar, parity)) {
+        record_status(status, NEST_ERR_TIMEOUT);
+        *reinterpret_cast<volatile int*>(abort_flag) = 1;
+    }
+}
+
 template <int DT, int NQ, int CPT>
 __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanArgs a)
 {
     constexpr int EPC = Elem<DT>::kPerChunk;
+    constexpr int PPC = EPC / 2;        // fp32 pairs per 16-byte chunk
     constexpr int NV = kScanRows * NQ;  // (row, query) dot products per stage
     constexpr int kLanesPerValue = 32 / NV;
     static_assert(NV <= 32 && (NV & (NV - 1)) == 0, "NV must be a power of two <= 32");
@@ -118,9 +140,9 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
 
     unsigned char* stages = smem;
     uint64_t* cand = reinterpret_cast<uint64_t*>(smem + (size_t)a.stages * a.stage_bytes);
-    float* partial = reinterpret_cast<float*>(cand + (size_t)NQ * a.cap);  // [2][warps][NV]
+    float* partial = reinterpret_cast<float*>(cand + (size_t)NQ * a.cap);  // [ring][warps][NV]
     ScanShared<NQ>& sh =
-        *reinterpret_cast<ScanShared<NQ>*>(partial + 2 * kConsumerWarps * NV);
+        *reinterpret_cast<ScanShared<NQ>*>(partial + kPartialRing * kConsumerWarps * NV);
 
     // ---- this CTA's queries and key rows [lo, hi)
     int64_t lo = 0, hi = 0;
@@ -144,18 +166,20 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
     }
     const int64_t nrows = hi - lo;
     const int nst = (int)((nrows + kScanRows - 1) / kScanRows);
+    auto rows_of = [&](int i) -> int {
+        const int64_t left = nrows - (int64_t)i * kScanRows;
+        return (int)(left < kScanRows ? left : kScanRows);
+    };
 
     if (tid == 0) {
         for (int s = 0; s < a.stages; ++s) {
             mbar_init(&sh.full[s], 1);
             mbar_init(&sh.empty[s], kConsumerWarps);
         }
-#pragma unroll
-        for (int b = 0; b < NQ; ++b) {
-            sh.cnt[b] = 0;
-            sh.thr[b] = kNoCandidate;
+        for (int s = 0; s < kPartialRing; ++s) {
+            mbar_init(&sh.pfull[s], kConsumers);
+            mbar_init(&sh.pempty[s], 32);
         }
-        sh.need_select[0] = sh.need_select[1] = 0;
         sh.abort = 0;
         sh.issued = 0;
         mbar_init_fence();
@@ -163,172 +187,207 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
     __syncthreads();
 
     // ---------------------------------------------------------------- producer
-    if (warp == kConsumerWarps) {
+    if (warp == kProducerWarp) {
         if (lane == 0 && nst > 0) {
             const uint64_t policy = l2_policy_evict_first();
             const unsigned char* src = static_cast<const unsigned char*>(a.K) + lo * a.row_bytes;
+            int slot = 0;
+            uint32_t phase = 0;  // phase of the slot's current round
             for (int i = 0; i < nst; ++i) {
-                const int slot = i % a.stages;
                 if (i >= a.stages) {
+                    wait_or_abort(&sh.empty[slot], phase ^ 1u, &sh.abort, a.status);
                     if (*reinterpret_cast<volatile int*>(&sh.abort)) break;
-                    if (!mbar_wait_bounded(&sh.empty[slot], ((i / a.stages) - 1) & 1)) {
-                        record_status(a.status, NEST_ERR_TIMEOUT);
-                        *reinterpret_cast<volatile int*>(&sh.abort) = 1;
-                        break;
-                    }
                 }
-                const int rows = (int)((nrows - (int64_t)i * kScanRows) < kScanRows ? (nrows - (int64_t)i * kScanRows) : kScanRows);
-                const uint32_t bytes = (uint32_t)rows * (uint32_t)a.row_bytes;
+                const uint32_t bytes = (uint32_t)rows_of(i) * (uint32_t)a.row_bytes;
                 mbar_arrive_expect_tx(&sh.full[slot], bytes);
                 bulk_copy_g2s_evict_first(stages + (size_t)slot * a.stage_bytes,
                                           src + (size_t)i * kScanRows * a.row_bytes, bytes,
                                           &sh.full[slot], policy);
                 *reinterpret_cast<volatile int*>(&sh.issued) = i + 1;
+                if (++slot == a.stages) {
+                    slot = 0;
+                    phase ^= 1u;
+                }
             }
         }
         return;
     }
 
     // ---------------------------------------------------------------- consumers
-    auto bar = [] { named_barrier(kBarConsumers, kConsumers); };
-
-    // Queries of the group, fixed column chunks of this thread, in registers.
-    float qf[CPT][NQ][EPC];
-    float qn[NQ];
+    if (warp < kConsumerWarps) {
+        // Queries of the group, fixed column chunks of this thread, as fp32 pairs.
+        float2 qf[CPT][NQ][PPC];
+        float qn[NQ];
 #pragma unroll
-    for (int b = 0; b < NQ; ++b) qn[b] = 0.f;
+        for (int b = 0; b < NQ; ++b) qn[b] = 0.f;
 #pragma unroll
-    for (int k = 0; k < CPT; ++k) {
-        const int c = tid + k * kConsumers;
+        for (int k = 0; k < CPT; ++k) {
+            const int c = tid + k * kConsumers;
 #pragma unroll
-        for (int b = 0; b < NQ; ++b) {
-            float x[EPC];
-            if (c < a.chunks && b < nqv) {
-                const uint4 v = ld_global_nc_v4(static_cast<const unsigned char*>(a.q) +
-                                                (size_t)(q0 + b) * a.row_bytes + (size_t)c * 16);
-                unpack_chunk<DT>(v, x);
-            } else {
+            for (int b = 0; b < NQ; ++b) {
+                float2 x[PPC];
+                if (c < a.chunks && b < nqv) {
+                    const uint4 v = ld_global_nc_v4(static_cast<const unsigned char*>(a.q) +
+                                                    (size_t)(q0 + b) * a.row_bytes + (size_t)c * 16);
+                    unpack_pairs<DT>(v, x);
+                } else {
 #pragma unroll
-                for (int e = 0; e < EPC; ++e) x[e] = 0.f;
-            }
+                    for (int p = 0; p < PPC; ++p) x[p] = make_float2(0.f, 0.f);
+                }
 #pragma unroll
-            for (int e = 0; e < EPC; ++e) {
-                qf[k][b][e] = x[e];
-                qn[b] = fmaf(x[e], x[e], qn[b]);
-            }
-        }
-    }
-    // ||q||^2 of each query, reduced over the CTA.
-#pragma unroll
-    for (int b = 0; b < NQ; ++b) {
-#pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) qn[b] += __shfl_xor_sync(~0u, qn[b], o);
-        if (lane == 0) partial[warp * NQ + b] = qn[b];
-    }
-    bar();
-    if (tid < NQ) {
-        float t = 0.f;
-        for (int w = 0; w < kConsumerWarps; ++w) t += partial[w * NQ + tid];
-        sh.qnorm[tid] = t;
-    }
-    bar();
-
-    // Key norms of a stage's rows, prefetched two stages ahead by warp 0.
-    const bool kn_lane = (warp == 0) && (lane < kScanRows);
-    auto load_kn = [&](int i) -> float {
-        const int64_t row = lo + (int64_t)i * kScanRows + lane;
-        return (kn_lane && i < nst && row < hi) ? __ldg(a.knorm + row) : 0.f;
-    };
-    float kn_cur = load_kn(0), kn_next = load_kn(1);
-
-    for (int i = 0; i < nst; ++i) {
-        const int slot = i % a.stages;
-        const int rows = (int)((nrows - (int64_t)i * kScanRows) < kScanRows ? (nrows - (int64_t)i * kScanRows) : kScanRows);
-        if (!*reinterpret_cast<volatile int*>(&sh.abort)) {
-            if (!mbar_wait_bounded(&sh.full[slot], (uint32_t)(i / a.stages) & 1u)) {
-                record_status(a.status, NEST_ERR_TIMEOUT);
-                *reinterpret_cast<volatile int*>(&sh.abort) = 1;
-            }
-        }
-        float acc[kScanRows][NQ];
-#pragma unroll
-        for (int rr = 0; rr < kScanRows; ++rr)
-#pragma unroll
-            for (int b = 0; b < NQ; ++b) acc[rr][b] = 0.f;
-        const unsigned char* st = stages + (size_t)slot * a.stage_bytes;
-#pragma unroll
-        for (int rr = 0; rr < kScanRows; ++rr) {
-            if (rr < rows) {
-#pragma unroll
-                for (int k = 0; k < CPT; ++k) {
-                    const int c = tid + k * kConsumers;
-                    if (c < a.chunks) {
-                        const uint4 v = *reinterpret_cast<const uint4*>(
-                            st + (size_t)rr * a.row_bytes + (size_t)c * 16);
-                        float x[EPC];
-                        unpack_chunk<DT>(v, x);
-#pragma unroll
-                        for (int b = 0; b < NQ; ++b)
-#pragma unroll
-                            for (int e = 0; e < EPC; ++e)
-                                acc[rr][b] = fmaf(qf[k][b][e], x[e], acc[rr][b]);
-                    }
+                for (int p = 0; p < PPC; ++p) {
+                    qf[k][b][p] = x[p];
+                    qn[b] = fmaf(x[p].x, x[p].x, qn[b]);
+                    qn[b] = fmaf(x[p].y, x[p].y, qn[b]);
                 }
             }
         }
+#pragma unroll
+        for (int b = 0; b < NQ; ++b) {
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) qn[b] += __shfl_xor_sync(~0u, qn[b], o);
+            if (lane == 0) sh.qnorm_part[warp][b] = qn[b];
+        }
+        named_barrier(kBarSetup, kConsumers + 32);
+
+        int slot = 0;
+        uint32_t phase = 0;
+        for (int i = 0; i < nst; ++i) {
+            const int rows = rows_of(i);
+            wait_or_abort(&sh.full[slot], phase, &sh.abort, a.status);
+            float2 acc[kScanRows][NQ];
+#pragma unroll
+            for (int rr = 0; rr < kScanRows; ++rr)
+#pragma unroll
+                for (int b = 0; b < NQ; ++b) acc[rr][b] = make_float2(0.f, 0.f);
+            const unsigned char* st = stages + (size_t)slot * a.stage_bytes;
+#pragma unroll
+            for (int rr = 0; rr < kScanRows; ++rr) {
+                if (rr < rows) {
+#pragma unroll
+                    for (int k = 0; k < CPT; ++k) {
+                        const int c = tid + k * kConsumers;
+                        if (c < a.chunks) {
+                            const uint4 v = *reinterpret_cast<const uint4*>(
+                                st + (size_t)rr * a.row_bytes + (size_t)c * 16);
+                            float2 x[PPC];
+                            unpack_pairs<DT>(v, x);
+#pragma unroll
+                            for (int b = 0; b < NQ; ++b)
+#pragma unroll
+                                for (int p = 0; p < PPC; ++p)
+                                    acc[rr][b] = __ffma2_rn(qf[k][b][p], x[p], acc[rr][b]);
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh.empty[slot]);
+            if (++slot == a.stages) {
+                slot = 0;
+                phase ^= 1u;
+            }
+
+            float v[NV];
+#pragma unroll
+            for (int rr = 0; rr < kScanRows; ++rr)
+#pragma unroll
+                for (int b = 0; b < NQ; ++b) v[rr * NQ + b] = acc[rr][b].x + acc[rr][b].y;
+            const float red = warp_reduce_scatter<NV>(v, lane);
+            const int ps = i & (kPartialRing - 1);
+            if (i >= kPartialRing)
+                wait_or_abort(&sh.pempty[ps], (uint32_t)((i / kPartialRing) - 1) & 1u, &sh.abort,
+                              a.status);
+            if ((lane & (kLanesPerValue - 1)) == 0)
+                partial[(ps * kConsumerWarps + warp) * NV + lane / kLanesPerValue] = red;
+            mbar_arrive(&sh.pfull[ps]);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- selector
+    named_barrier(kBarSetup, kConsumers + 32);
+    float qnorm[NQ];
+#pragma unroll
+    for (int b = 0; b < NQ; ++b) {
+        float t = 0.f;
+        for (int w = 0; w < kConsumerWarps; ++w) t += sh.qnorm_part[w][b];
+        qnorm[b] = t;
+    }
+    if (lane < NQ) {
+        sh.cnt[lane] = 0;
+        sh.thr[lane] = kNoCandidate;
+    }
+    __syncwarp();
+    int cnt[NQ];
+#pragma unroll
+    for (int b = 0; b < NQ; ++b) cnt[b] = 0;
+
+    // Key norms of a stage's rows, prefetched two stages ahead (lanes < kScanRows).
+    auto load_kn = [&](int i) -> float {
+        const int64_t row = lo + (int64_t)i * kScanRows + lane;
+        return (lane < kScanRows && i < nst && row < hi) ? __ldg(a.knorm + row) : 0.f;
+    };
+    float kn_cur = load_kn(0), kn_next = load_kn(1);
+    const int rr = lane / NQ, b = lane % NQ;
+    float qnorm_b = 0.f;  // ||q_b||^2 of this lane's query (no dynamic register indexing)
+#pragma unroll
+    for (int qb = 0; qb < NQ; ++qb)
+        if (b == qb) qnorm_b = qnorm[qb];
+
+    for (int i = 0; i < nst; ++i) {
+        const int ps = i & (kPartialRing - 1);
+        const int rows = rows_of(i);
+        wait_or_abort(&sh.pfull[ps], (uint32_t)(i / kPartialRing) & 1u, &sh.abort, a.status);
+        const float kn = __shfl_sync(~0u, kn_cur, rr & (kScanRows - 1));
+        bool accept = false;
+        uint64_t key = 0;
+        if (lane < NV) {
+            float dot = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) dot += partial[(ps * kConsumerWarps + w) * NV + lane];
+            float dist = fmaf(-2.f, dot, qnorm_b + kn);
+            dist = (dist <= 0.f) ? 0.f : dist;  // NaN stays NaN and sorts last
+            const int64_t row = lo + (int64_t)i * kScanRows + rr;
+            key = ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)row;
+            accept = (rr < rows) && (b < nqv) && (key <= sh.thr[b]);
+        }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sh.empty[slot]);
-
-        float v[NV];
+        mbar_arrive(&sh.pempty[ps]);
+        const uint32_t bal = __ballot_sync(~0u, accept);
+        bool full = false;
 #pragma unroll
-        for (int rr = 0; rr < kScanRows; ++rr)
+        for (int qb = 0; qb < NQ; ++qb) {
+            const uint32_t qm = bal & query_lanes<NQ, NV>(qb);
+            if (accept && b == qb) cand[(size_t)qb * a.cap + cnt[qb] + __popc(qm & lanemask_lt())] = key;
+            cnt[qb] += __popc(qm);
+            full |= cnt[qb] > a.cap - kScanRows;
+        }
+        kn_cur = kn_next;
+        kn_next = load_kn(i + 2);
+        if (full) {
+            __syncwarp();
+            if (lane == 0) {
 #pragma unroll
-            for (int b = 0; b < NQ; ++b) v[rr * NQ + b] = acc[rr][b];
-        const float red = warp_reduce_scatter<NV>(v, lane);
-        if ((lane & (kLanesPerValue - 1)) == 0)
-            partial[((i & 1) * kConsumerWarps + warp) * NV + lane / kLanesPerValue] = red;
-        bar();
-
-        if (sh.need_select[i & 1]) select_smallest<kConsumers, NQ>(cand, a.cap, sh.cnt, sh.thr, a.r, sh.sel, tid, bar);
-
-        if (warp == 0) {
-            const int rr = lane / NQ, b = lane % NQ;
-            const float kn = __shfl_sync(~0u, kn_cur, rr & (kScanRows - 1));
-            bool accept = false;
-            uint64_t key = 0;
-            if (lane < NV) {
-                float dot = 0.f;
-#pragma unroll
-                for (int w = 0; w < kConsumerWarps; ++w)
-                    dot += partial[((i & 1) * kConsumerWarps + w) * NV + lane];
-                float dist = fmaf(-2.f, dot, sh.qnorm[b] + kn);
-                dist = (dist <= 0.f) ? 0.f : dist;  // NaN stays NaN and sorts last
-                const int64_t row = lo + (int64_t)i * kScanRows + rr;
-                key = ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)row;
-                accept = (rr < rows) && (b < nqv) && (key <= sh.thr[b]);
+                for (int qb = 0; qb < NQ; ++qb) sh.cnt[qb] = cnt[qb];
             }
-            const uint32_t bal = __ballot_sync(~0u, accept);
-            bool full = false;
+            __syncwarp();
+            select_smallest<32, NQ>(cand, a.cap, sh.cnt, sh.thr, a.r, sh.sel, lane,
+                                    [] { __syncwarp(); });
 #pragma unroll
-            for (int qb = 0; qb < NQ; ++qb) {
-                const uint32_t qm = bal & query_lanes<NQ, NV>(qb);
-                const int base = sh.cnt[qb];
-                if (accept && b == qb) cand[(size_t)qb * a.cap + base + __popc(qm & lanemask_lt())] = key;
-                const int nc = base + __popc(qm);
-                full |= nc > a.cap - kScanRows;
-                __syncwarp();
-                if (lane == 0) sh.cnt[qb] = nc;
-            }
-            if (lane == 0) sh.need_select[(i + 1) & 1] = full ? 1 : 0;
-            kn_cur = kn_next;
-            kn_next = load_kn(i + 2);
+            for (int qb = 0; qb < NQ; ++qb) cnt[qb] = sh.cnt[qb];
         }
     }
-    bar();
-    select_smallest<kConsumers, NQ>(cand, a.cap, sh.cnt, sh.thr, a.r, sh.sel, tid, bar);
+    __syncwarp();
+    if (lane == 0) {
+#pragma unroll
+        for (int qb = 0; qb < NQ; ++qb) sh.cnt[qb] = cnt[qb];
+    }
+    __syncwarp();
+    select_smallest<32, NQ>(cand, a.cap, sh.cnt, sh.thr, a.r, sh.sel, lane, [] { __syncwarp(); });
 
     // Copies still in flight after an abort must land before the CTA exits.
-    if (tid == 0 && *reinterpret_cast<volatile int*>(&sh.abort)) {
+    if (lane == 0 && *reinterpret_cast<volatile int*>(&sh.abort)) {
         const int issued = *reinterpret_cast<volatile int*>(&sh.issued);
         for (int i = max(0, issued - a.stages); i < issued; ++i)
             (void)mbar_wait_bounded(&sh.full[i % a.stages], (uint32_t)(i / a.stages) & 1u);
@@ -336,10 +395,10 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
 
     uint64_t* out = a.cand + (size_t)item * NQ * a.r;
 #pragma unroll
-    for (int b = 0; b < NQ; ++b) {
-        const int n = sh.cnt[b];
-        for (int j = tid; j < a.r; j += kConsumers)
-            out[(size_t)b * a.r + j] = j < n ? cand[(size_t)b * a.cap + j] : kNoCandidate;
+    for (int qb = 0; qb < NQ; ++qb) {
+        const int n = sh.cnt[qb];
+        for (int j = lane; j < a.r; j += 32)
+            out[(size_t)qb * a.r + j] = j < n ? cand[(size_t)qb * a.cap + j] : kNoCandidate;
     }
 }
 
@@ -379,7 +438,8 @@ cudaError_t launch_nq(const ScanPlan& p, const ScanArgs& a, cudaStream_t stream)
 template <int NQ>
 size_t fixed_smem(int cap)
 {
-    return (size_t)NQ * cap * sizeof(uint64_t) + 2 * kConsumerWarps * kScanRows * NQ * sizeof(float) +
+    return (size_t)NQ * cap * sizeof(uint64_t) +
+           (size_t)kPartialRing * kConsumerWarps * kScanRows * NQ * sizeof(float) +
            sizeof(ScanShared<NQ>) + 128;
 }
 
@@ -390,7 +450,9 @@ bool scan_plan_smem(int dtype, int nq, int cpt, int r, int row_bytes, size_t sme
 {
     if (dtype != NEST_F32 && dtype != NEST_BF16) return false;
     if (cpt != 1 && cpt != 2 && cpt != 4) return false;
-    const int cap = r < 64 ? r + 64 : 2 * r;
+    // r kept candidates plus room to append before a trim; trims are cheap
+    // enough that 512 slots of room suffice once r is large.
+    const int cap = r < 64 ? r + 64 : (r < 512 ? 2 * r : r + 512);
     size_t fixed;
     switch (nq) {
     case 1: fixed = fixed_smem<1>(cap); break;

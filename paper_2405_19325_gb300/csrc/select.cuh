@@ -75,8 +75,8 @@ __device__ __forceinline__ void select_smallest(uint64_t* buf, int stride, int* 
             }
         }
         bar();
-        if (warp < NQ && !s.done[warp]) {
-            const int b = warp;
+        for (int b = warp; b < NQ; b += NT / 32) {
+            if (s.done[b]) continue;
             uint32_t h[8];
             uint32_t local = 0;
 #pragma unroll
