@@ -55,7 +55,7 @@ typedef enum nest_status {
     NEST_ERR_OOM = 4,          /* device allocation failed */
     NEST_ERR_CUDA = 5,         /* a CUDA runtime call failed */
     NEST_ERR_VALUE_RANGE = 6,  /* token id outside [0, vocab) or key index outside [0, N) */
-    NEST_ERR_OVERFLOW = 7,     /* reserved: a bounded device buffer overflowed */
+    NEST_ERR_OVERFLOW = 7,     /* a search needs more than a fixed-size scratch buffer holds */
     NEST_ERR_TIMEOUT = 8,      /* a device-side wait gave up */
     NEST_ERR_UNSUPPORTED = 9   /* shape outside what the kernels handle */
 } nest_status_t;
@@ -126,6 +126,38 @@ NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_
 NEST_API nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
                               const int64_t* seg_off, float* s_out, int64_t* idx_out,
                               void* stream);
+
+/*
+ * nest_knn_search without any device allocation (the paper has no
+ * counterpart: this is a deployment variant of the search above).
+ *
+ * nest_knn_search places its candidate lists in scratch memory that the
+ * handle allocates with cudaMalloc on first use and re-allocates when a
+ * larger search comes; cudaMalloc and cudaFree synchronize the device and
+ * draw on memory that a framework's own allocator may already own.  Callers
+ * that must not allocate -- for example a serving loop that may never stall
+ * the device, or an application whose allocator owns all device memory --
+ * call this instead.  It runs the same kernels and writes the same outputs,
+ * with the candidate lists in one fixed 8 MiB array compiled into the
+ * library, which every GPU that loads the library holds until the process
+ * exits.
+ *
+ *   Arguments, outputs and device-side errors are those of nest_knn_search.
+ *   Returns NEST_ERR_OVERFLOW, before launching anything, when the search
+ *   needs more than the 2^20 candidate words (8 MiB) of the array; the
+ *   decode and second-stage workloads need far less (1M keys, B = 4,
+ *   r = 1024: about 0.65M words).
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress) with that device current; make that first call
+ *   before any stream capture.
+ *   All calls on a device share the one array and it keeps what the last
+ *   call left in it (no call relies on it starting at zero): calls that
+ *   overlap on the GPU, from different streams or threads, race with each
+ *   other and must be serialized by the caller.
+ */
+NEST_API nest_status_t nest_knn_search_static(nest_datastore_t* ds, const void* q, int32_t B,
+                                              int32_t r, const int64_t* seg_off, float* s_out,
+                                              int64_t* idx_out, void* stream);
 
 /*
  * Eq. 2 and Eq. 3 for each query row b < B:

@@ -457,3 +457,82 @@ const char* nest_status_string(nest_status_t s)
 int32_t nest_version(void) { return 100; }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- caller-provided scratch
+// Used by the allocation-free search entry point (noalloc.cu): the same plan
+// and kernels as nest_knn_search, with the candidate lists placed in memory
+// the caller of these helpers owns.
+namespace nest {
+
+nest_status_t search_scratch_words(const nest_datastore* ds, int32_t B, int32_t r, bool ragged,
+                                   size_t* words)
+{
+    SearchPlan sp;
+    nest_status_t st = plan_search(ds, B, r, ragged, &sp);
+    if (st != NEST_OK) return st;
+    *words = sp.cand_words + sp.level_words;
+    return NEST_OK;
+}
+
+nest_status_t search_with_scratch(nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                                  const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                                  uint64_t* scratch, size_t scratch_words, cudaStream_t stream)
+{
+    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st != NEST_OK) return st;
+    SearchPlan sp;
+    st = plan_search(ds, B, r, seg_off != nullptr, &sp);
+    if (st != NEST_OK) return st;
+    if (sp.cand_words + sp.level_words > scratch_words) return NEST_ERR_OVERFLOW;
+    uint64_t* regionA = scratch;
+    uint64_t* regionB = scratch + sp.cand_words;
+
+    ScanArgs sa{};
+    sa.K = ds->K;
+    sa.knorm = ds->knorm;
+    sa.q = q;
+    sa.seg_off = seg_off;
+    sa.cand = regionA;
+    sa.status = ds->status;
+    sa.N = ds->N;
+    sa.row_bytes = ds->row_bytes;
+    sa.chunks = ds->row_bytes / 16;
+    sa.B = B;
+    sa.r = r;
+    sa.cap = sp.scan.cap;
+    sa.parts = sp.scan.parts;
+    sa.stages = sp.scan.stages;
+    sa.stage_bytes = sp.scan.stage_bytes;
+    cudaError_t e = launch_scan(ds->dtype, sp.scan, sa, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
+
+    MergeArgs ma{};
+    ma.in = regionA;
+    ma.list_stride = (int64_t)sp.scan.nq * r;
+    ma.nq_in = sp.scan.nq;
+    ma.lists = sp.scan.parts;
+    ma.B = B;
+    ma.r = r;
+    ma.s_out = s_out;
+    ma.idx_out = idx_out;
+    bool into_b = true;
+    for (;;) {
+        ma.per_cta = std::min(merge_lists_per_cta(r), ma.lists);
+        const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
+        const bool last = groups == 1;
+        ma.out = into_b ? regionB : regionA;
+        e = launch_merge(ma, last, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        ++ds->launches;
+        if (last) break;
+        ma.in = ma.out;
+        ma.list_stride = r;
+        ma.nq_in = 1;
+        ma.lists = groups;
+        into_b = !into_b;
+    }
+    return NEST_OK;
+}
+
+}  // namespace nest

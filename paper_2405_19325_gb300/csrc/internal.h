@@ -110,4 +110,14 @@ struct MixArgs {
 
 cudaError_t launch_mix(const MixArgs& args, cudaStream_t stream);
 
+// ---------------------------------------------------------------- api.cu, for noalloc.cu
+// Scratch words (64-bit) a search of this shape needs; no allocation, no launch.
+nest_status_t search_scratch_words(const nest_datastore_t* ds, int32_t B, int32_t r, bool ragged,
+                                   size_t* words);
+// nest_knn_search with the candidate lists in caller-provided device memory
+// of scratch_words words; NEST_ERR_OVERFLOW if the search needs more.
+nest_status_t search_with_scratch(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                                  const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                                  uint64_t* scratch, size_t scratch_words, cudaStream_t stream);
+
 }  // namespace nest

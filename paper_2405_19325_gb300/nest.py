@@ -34,6 +34,7 @@ SIGNATURES = {
     "nest_datastore_destroy": (ctypes.c_int, [_P]),
     "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
     "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
+    "nest_knn_search_static": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_mix": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _P, _P, _P]),
     "nest_knn_mix_rrc": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _F, _P, _P, _P, _P]),
     "nest_knn_step": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _F, _F, _P, _P, _P, _P, _P]),
