@@ -6,6 +6,8 @@
 #include <new>
 #include <vector>
 
+#include <cudaTypedefs.h>
+
 #include "internal.h"
 
 using namespace nest;
@@ -21,6 +23,8 @@ struct nest_datastore {
     int device = 0;
     int num_sms = 1;
     size_t smem_optin = 0;
+    bool tc = false;         // bf16 keys with a TMA tensor map: tensor-core scan
+    CUtensorMap keys_map;  // TMA map of K (type is 64-byte aligned)
     float* knorm = nullptr;  // owned: ||k_i||^2, N floats
     int* status = nullptr;   // owned: device status word
     uint64_t* scratch = nullptr;  // owned: candidate lists of the search
@@ -49,9 +53,13 @@ cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
 
 int element_size(int dtype) { return dtype == NEST_BF16 ? 2 : 4; }
 
-// Search layout chosen for a call: the scan kernel's plan and the merge tree.
+// Search layout chosen for a call: which scan kernel, its plan, and the
+// candidate words of the scan output and of the merge levels.
 struct SearchPlan {
+    bool tc;       // tensor-core scan (bf16) or CUDA-core scan
     ScanPlan scan;
+    TcPlan tcp;
+    int nq, groups, parts;
     size_t cand_words;   // scan output: groups * parts * nq * r
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
 };
@@ -78,25 +86,99 @@ int choose_parts(int groups, int64_t keys_per_group, int num_sms, bool ragged)
     return best;
 }
 
+int ceil_pow2(int x)
+{
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
 nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, SearchPlan* sp)
 {
-    const int chunks = ds->row_bytes / 16;
-    const int cpt = chunks <= 256 ? 1 : (chunks <= 512 ? 2 : 4);
-    int nq = ragged ? 1 : (B >= 3 ? 4 : B);
-    ScanPlan p{};
-    while (!scan_plan_smem(ds->dtype, nq, cpt, r, ds->row_bytes, ds->smem_optin, &p)) {
-        if (nq == 1) return NEST_ERR_UNSUPPORTED;
-        nq /= 2;
+    sp->tc = false;
+    const int64_t keys_per_group_full = ds->N;
+    if (ds->tc) {
+        int nq = ragged ? 1 : ceil_pow2(std::min(B, 16));
+        TcPlan tp{};
+        bool ok = false;
+        for (;;) {
+            if (tc_plan_smem(nq, r, ds->smem_optin, &tp)) {
+                ok = true;
+                break;
+            }
+            if (nq == 1) break;
+            nq /= 2;
+        }
+        if (ok) {
+            tp.groups = ragged ? B : (B + nq - 1) / nq;
+            const int64_t keys_per_group = ragged ? (ds->N + B - 1) / B : keys_per_group_full;
+            tp.parts = choose_parts(tp.groups, keys_per_group, ds->num_sms, ragged);
+            sp->tc = true;
+            sp->tcp = tp;
+            sp->nq = nq;
+            sp->groups = tp.groups;
+            sp->parts = tp.parts;
+        }
     }
-    p.groups = ragged ? B : (B + nq - 1) / nq;
-    const int64_t keys_per_group = ragged ? (ds->N + B - 1) / B : ds->N;
-    p.parts = choose_parts(p.groups, keys_per_group, ds->num_sms, ragged);
-    sp->scan = p;
-    sp->cand_words = (size_t)p.groups * p.parts * p.nq * r;
+    if (!sp->tc) {
+        const int chunks = ds->row_bytes / 16;
+        const int cpt = chunks <= 256 ? 1 : (chunks <= 512 ? 2 : 4);
+        int nq = ragged ? 1 : (B >= 3 ? 4 : B);
+        ScanPlan p{};
+        while (!scan_plan_smem(ds->dtype, nq, cpt, r, ds->row_bytes, ds->smem_optin, &p)) {
+            if (nq == 1) return NEST_ERR_UNSUPPORTED;
+            nq /= 2;
+        }
+        p.groups = ragged ? B : (B + nq - 1) / nq;
+        const int64_t keys_per_group = ragged ? (ds->N + B - 1) / B : keys_per_group_full;
+        p.parts = choose_parts(p.groups, keys_per_group, ds->num_sms, ragged);
+        sp->scan = p;
+        sp->nq = p.nq;
+        sp->groups = p.groups;
+        sp->parts = p.parts;
+    }
+    sp->cand_words = (size_t)sp->groups * sp->parts * sp->nq * r;
     const int per = merge_lists_per_cta(r);
-    const int lvl1 = (p.parts + per - 1) / per;
+    const int lvl1 = (sp->parts + per - 1) / per;
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
     return NEST_OK;
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            (void)cudaGetLastError();
+            p = nullptr;
+        }
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }();
+    return fn;
+}
+
+// 2-D bf16 tensor map over rows x d (row stride d * 2 bytes), box of
+// box_rows rows x 64 columns, 128-byte swizzle; rows and columns outside
+// the tensor read as zero.
+bool encode_bf16_rows(CUtensorMap* map, const void* base, int64_t rows, int32_t d, int box_rows,
+                      bool keys)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    const cuuint32_t elem[2] = {1, 1};
+    const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                           strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B,
+                           keys ? CU_TENSOR_MAP_L2_PROMOTION_L2_256B : CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
 }
 
 nest_status_t ensure_scratch(nest_datastore* ds, size_t words)
@@ -164,47 +246,70 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
     return NEST_OK;
 }
 
-nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
-                         const int64_t* seg_off, float* s_out, int64_t* idx_out,
-                         cudaStream_t stream)
+// Plan, check the scratch, launch the scan and the merge tree.  The scratch
+// (64-bit words) is the handle's own or the caller's; timing events are
+// recorded around the scan when `timed`.
+nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                            const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                            uint64_t* scratch, size_t scratch_words, bool timed,
+                            cudaStream_t stream)
 {
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
     if (st != NEST_OK) return st;
-    st = ensure_scratch(ds, sp.cand_words + sp.level_words);
-    if (st != NEST_OK) return st;
+    if (sp.cand_words + sp.level_words > scratch_words) return NEST_ERR_OVERFLOW;
+    uint64_t* regionA = scratch;
+    uint64_t* regionB = scratch + sp.cand_words;
 
-    uint64_t* regionA = ds->scratch;
-    uint64_t* regionB = ds->scratch + sp.cand_words;
-
-    ScanArgs sa{};
-    sa.K = ds->K;
-    sa.knorm = ds->knorm;
-    sa.q = q;
-    sa.seg_off = seg_off;
-    sa.cand = regionA;
-    sa.status = ds->status;
-    sa.N = ds->N;
-    sa.row_bytes = ds->row_bytes;
-    sa.chunks = ds->row_bytes / 16;
-    sa.B = B;
-    sa.r = r;
-    sa.cap = sp.scan.cap;
-    sa.parts = sp.scan.parts;
-    sa.stages = sp.scan.stages;
-    sa.stage_bytes = sp.scan.stage_bytes;
-
-    if (ds->timing && (st = record_event(ds, stream)) != NEST_OK) return st;
-    cudaError_t e = launch_scan(ds->dtype, sp.scan, sa, stream);
+    cudaError_t e;
+    if (sp.tc) {
+        CUtensorMap qmap;
+        if (!encode_bf16_rows(&qmap, q, B, ds->d, 16, false)) return NEST_ERR_CUDA;
+        TcScanArgs ta{};
+        ta.knorm = ds->knorm;
+        ta.q = q;
+        ta.seg_off = seg_off;
+        ta.cand = regionA;
+        ta.status = ds->status;
+        ta.N = ds->N;
+        ta.d = ds->d;
+        ta.B = B;
+        ta.r = r;
+        ta.cap = sp.tcp.cap;
+        ta.parts = sp.tcp.parts;
+        ta.stages = sp.tcp.stages;
+        ta.kchunks = (ds->d + 63) / 64;
+        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+        e = launch_tc_scan(sp.tcp, ds->keys_map, qmap, ta, stream);
+    } else {
+        ScanArgs sa{};
+        sa.K = ds->K;
+        sa.knorm = ds->knorm;
+        sa.q = q;
+        sa.seg_off = seg_off;
+        sa.cand = regionA;
+        sa.status = ds->status;
+        sa.N = ds->N;
+        sa.row_bytes = ds->row_bytes;
+        sa.chunks = ds->row_bytes / 16;
+        sa.B = B;
+        sa.r = r;
+        sa.cap = sp.scan.cap;
+        sa.parts = sp.scan.parts;
+        sa.stages = sp.scan.stages;
+        sa.stage_bytes = sp.scan.stage_bytes;
+        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+        e = launch_scan(ds->dtype, sp.scan, sa, stream);
+    }
     if (e != cudaSuccess) return from_cuda(e);
     ++ds->launches;
-    if (ds->timing && (st = record_event(ds, stream)) != NEST_OK) return st;
+    if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
 
     MergeArgs ma{};
     ma.in = regionA;
-    ma.list_stride = (int64_t)sp.scan.nq * r;
-    ma.nq_in = sp.scan.nq;
-    ma.lists = sp.scan.parts;
+    ma.list_stride = (int64_t)sp.nq * r;
+    ma.nq_in = sp.nq;
+    ma.lists = sp.parts;
     ma.B = B;
     ma.r = r;
     ma.s_out = s_out;
@@ -226,6 +331,19 @@ nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r
         into_b = !into_b;
     }
     return NEST_OK;
+}
+
+nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                         const int64_t* seg_off, float* s_out, int64_t* idx_out,
+                         cudaStream_t stream)
+{
+    SearchPlan sp;
+    nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
+    if (st != NEST_OK) return st;
+    st = ensure_scratch(ds, sp.cand_words + sp.level_words);
+    if (st != NEST_OK) return st;
+    return launch_search(ds, q, B, r, seg_off, s_out, idx_out, ds->scratch, ds->scratch_words,
+                         ds->timing, stream);
 }
 
 nest_status_t run_mix(nest_datastore* ds, const float* s_in, const int64_t* idx_in,
@@ -310,6 +428,9 @@ nest_status_t nest_datastore_create(const void* K, const int32_t* V, int64_t N, 
         return e == cudaErrorMemoryAllocation ? NEST_ERR_OOM : NEST_ERR_CUDA;
     }
     ds->launches = 2;
+    // Tensor-core scan: bf16 keys whose row indices fit TMA's 32-bit coordinates.
+    if (dtype == NEST_BF16 && N <= (int64_t)0x7FFFFF00)
+        ds->tc = encode_bf16_rows(&ds->keys_map, K, N, d, kTcTileKeys, true);
     if (host_status != 0) {
         nest_datastore_destroy(ds);
         return static_cast<nest_status_t>(host_status);
@@ -480,59 +601,8 @@ nest_status_t search_with_scratch(nest_datastore* ds, const void* q, int32_t B, 
 {
     nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
     if (st != NEST_OK) return st;
-    SearchPlan sp;
-    st = plan_search(ds, B, r, seg_off != nullptr, &sp);
-    if (st != NEST_OK) return st;
-    if (sp.cand_words + sp.level_words > scratch_words) return NEST_ERR_OVERFLOW;
-    uint64_t* regionA = scratch;
-    uint64_t* regionB = scratch + sp.cand_words;
-
-    ScanArgs sa{};
-    sa.K = ds->K;
-    sa.knorm = ds->knorm;
-    sa.q = q;
-    sa.seg_off = seg_off;
-    sa.cand = regionA;
-    sa.status = ds->status;
-    sa.N = ds->N;
-    sa.row_bytes = ds->row_bytes;
-    sa.chunks = ds->row_bytes / 16;
-    sa.B = B;
-    sa.r = r;
-    sa.cap = sp.scan.cap;
-    sa.parts = sp.scan.parts;
-    sa.stages = sp.scan.stages;
-    sa.stage_bytes = sp.scan.stage_bytes;
-    cudaError_t e = launch_scan(ds->dtype, sp.scan, sa, stream);
-    if (e != cudaSuccess) return from_cuda(e);
-    ++ds->launches;
-
-    MergeArgs ma{};
-    ma.in = regionA;
-    ma.list_stride = (int64_t)sp.scan.nq * r;
-    ma.nq_in = sp.scan.nq;
-    ma.lists = sp.scan.parts;
-    ma.B = B;
-    ma.r = r;
-    ma.s_out = s_out;
-    ma.idx_out = idx_out;
-    bool into_b = true;
-    for (;;) {
-        ma.per_cta = std::min(merge_lists_per_cta(r), ma.lists);
-        const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
-        const bool last = groups == 1;
-        ma.out = into_b ? regionB : regionA;
-        e = launch_merge(ma, last, stream);
-        if (e != cudaSuccess) return from_cuda(e);
-        ++ds->launches;
-        if (last) break;
-        ma.in = ma.out;
-        ma.list_stride = r;
-        ma.nq_in = 1;
-        ma.lists = groups;
-        into_b = !into_b;
-    }
-    return NEST_OK;
+    return launch_search(ds, q, B, r, seg_off, s_out, idx_out, scratch, scratch_words, false,
+                         stream);
 }
 
 }  // namespace nest

@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "../../include/nest.h"
@@ -66,6 +67,41 @@ bool scan_plan_smem(int dtype, int nq, int cpt, int r, int row_bytes, size_t sme
                     ScanPlan* plan);
 cudaError_t launch_scan(int dtype, const ScanPlan& plan, const ScanArgs& args,
                         cudaStream_t stream);
+
+// ---------------------------------------------------------------- tc_scan.cu
+// Tensor-core (tcgen05) distance scan with fused per-CTA top-r, bf16 keys.
+constexpr int kTcThreads = 192;  // producer warp, MMA warp, 4 epilogue warps
+constexpr int kTcTileKeys = 128;  // keys per tensor-core tile
+
+struct TcPlan {
+    int nq;       // queries per CTA (1, 2, 4, 8 or 16; the MMA always has 16 columns)
+    int cap;      // candidate buffer entries per query
+    int stages;   // pipeline depth (18 KiB per stage)
+    int groups;   // query groups
+    int parts;    // key-range parts per group (whole 128-key tiles)
+    size_t smem;  // dynamic shared memory of one CTA
+};
+
+struct TcScanArgs {
+    const float* knorm;
+    const void* q;
+    const int64_t* seg_off;  // nullptr: full scan
+    uint64_t* cand;          // [groups * parts][nq][r]
+    int* status;
+    int64_t N;
+    int32_t d;
+    int32_t B;
+    int32_t r;
+    int32_t cap;
+    int32_t parts;
+    int32_t stages;
+    int32_t kchunks;  // ceil(d / 64)
+};
+
+int tc_cap(int r);
+bool tc_plan_smem(int nq, int r, size_t smem_limit, TcPlan* plan);
+cudaError_t launch_tc_scan(const TcPlan& plan, const CUtensorMap& keys, const CUtensorMap& queries,
+                           const TcScanArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- merge.cu
 // Merge candidate lists of each query into its top r.
