@@ -254,6 +254,20 @@ def run_reference(args, w, world, rank):
     print(json.dumps(line), flush=True)
 
 
+# DRAM bytes (read + write) per launch of the dominant kernel, from the ncu
+# capture summarised in profiles/tc_scan_decode_d4096_B4.md: 65,536-key case
+# scaled to the default 1,048,576 keys (reads x16, per-CTA writes unscaled).
+# Only valid for that kernel version on the default decode workload.
+DECODE_TC_SCAN_TRAFFIC = 537.27e6 * 16 + 3.05e6
+
+
+def dram_traffic(w, args, kernel):
+    if (w.name == "decode" and kernel == "tc_scan_kernel" and args.N is None
+            and args.B is None):
+        return DECODE_TC_SCAN_TRAFFIC
+    return None
+
+
 def config_of(w, x):
     B = x.q.shape[0]
     return {"workload": w.name, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
@@ -325,8 +339,10 @@ def main():
     scan_avg_ms = scan_ms / max(1, scan_n)
     hbm_peak, peak_kind = peaks()
     achieved = alg_bytes / (scan_avg_ms / 1e3) / 1e9
+    kernel = "tc_scan_kernel" if w.dtype == "bf16" else "scan_topr_kernel"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                "frac": achieved / hbm_peak, "traffic": None, "kernel": "scan_topr_kernel",
+                "frac": achieved / hbm_peak, "traffic": dram_traffic(w, args, kernel),
+                "kernel": kernel,
                 "peak_kind": peak_kind, "alg_bytes_per_launch": alg_bytes,
                 "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
 
