@@ -62,6 +62,14 @@ struct SearchPlan {
     int nq, groups, parts;
     size_t cand_words;   // scan output: groups * parts * nq * r
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
+    // Large query batches (tc_wide.cu): sample pass + thresholded pass.
+    bool wide;
+    WidePlan wps, wpm;        // sample pass, main pass
+    int64_t stride;           // sample = every stride-th key
+    int64_t sample_rows;
+    bool single_pass;         // the sample is the whole datastore
+    int64_t cap_s, cap_m;     // list capacities per query
+    size_t off_cnt, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
 };
 
 // Parts per query group.  Time ~ waves * (work per part + fixed cost per part),
@@ -141,6 +149,36 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
     const int per = merge_lists_per_cta(r);
     const int lvl1 = (sp->parts + per - 1) / per;
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
+    sp->wide = false;
+    // More queries than one CTA can keep lists for: stream the keys once per
+    // group of up to 256 queries against sampled admission thresholds.
+    if (sp->tc && !ragged && sp->groups > 1) {
+        const int nm = B >= 256 ? 256 : std::max(16, ceil_pow2(B));
+        WidePlan wp{};
+        if (wide_plan_smem(nm, ds->smem_optin, &wp)) {
+            wp.groups = (B + nm - 1) / nm;
+            const int64_t target = std::max<int64_t>(65536, 256LL * r);
+            sp->stride = std::max<int64_t>(1, ds->N / target);
+            sp->sample_rows = ds->N / sp->stride;
+            sp->single_pass = sp->stride == 1;
+            sp->wps = wp;
+            sp->wps.parts = choose_parts(wp.groups, sp->sample_rows, ds->num_sms, false);
+            sp->wpm = wp;
+            sp->wpm.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
+            sp->cap_s = sp->sample_rows;
+            const int64_t expect = (ds->N * (int64_t)r + sp->sample_rows - 1) / sp->sample_rows;
+            sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect));
+            sp->off_cnt = 0;  // 2 * B int32 counters
+            sp->off_cand_s = (size_t)B;
+            sp->off_s_s = sp->off_cand_s + (size_t)B * sp->cap_s;
+            sp->off_i_s = sp->off_s_s + ((size_t)B * r + 1) / 2;
+            sp->off_cand_m = sp->off_i_s + (size_t)B * r;
+            sp->wide_words = sp->single_pass ? sp->off_s_s : sp->off_cand_m + (size_t)B * sp->cap_m;
+            sp->wide = true;
+            sp->cand_words = sp->wide_words;
+            sp->level_words = 0;
+        }
+    }
     return NEST_OK;
 }
 
@@ -165,12 +203,12 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
 // box_rows rows x 64 columns, 128-byte swizzle; rows and columns outside
 // the tensor read as zero.
 bool encode_bf16_rows(CUtensorMap* map, const void* base, int64_t rows, int32_t d, int box_rows,
-                      bool keys)
+                      bool keys, int64_t row_step = 1)
 {
     auto enc = tensor_map_encoder();
     if (!enc) return false;
     const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
-    const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+    const cuuint64_t strides[1] = {(cuuint64_t)d * 2 * (cuuint64_t)row_step};
     const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
     const cuuint32_t elem[2] = {1, 1};
     const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
@@ -246,6 +284,103 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
     return NEST_OK;
 }
 
+// Large query batches: [sample pass, selection of the sample,] thresholded
+// pass over all keys, exact selection of the survivors.
+nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* q, int32_t B,
+                          int32_t r, float* s_out, int64_t* idx_out, uint64_t* scratch, bool timed,
+                          cudaStream_t stream)
+{
+    nest_status_t st;
+    int32_t* cnt = reinterpret_cast<int32_t*>(scratch + sp.off_cnt);
+    cudaError_t e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * 2 * (size_t)B, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    CUtensorMap qmap;
+    if (!encode_bf16_rows(&qmap, q, B, ds->d, sp.wpm.nm, false)) return NEST_ERR_CUDA;
+
+    WideArgs wa{};
+    wa.knorm = ds->knorm;
+    wa.q = q;
+    wa.status = ds->status;
+    wa.r = r;
+    wa.d = ds->d;
+    wa.B = B;
+    wa.groups = sp.wpm.groups;
+    wa.stages = sp.wpm.stages;
+    wa.kchunks = (ds->d + 63) / 64;
+
+    GselectArgs ga{};
+    ga.r = r;
+    ga.B = B;
+
+    if (sp.single_pass) {
+        // the "sample" is every key: its exact r nearest are the answer
+        wa.s_sample = nullptr;
+        wa.cand = scratch + sp.off_cand_s;
+        wa.cnt = cnt;
+        wa.cap = sp.cap_s;
+        wa.N = ds->N;
+        wa.parts = sp.wpm.parts;
+        wa.key_stride = 1;
+        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+        e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+        ga.cand = wa.cand;
+        ga.cnt = cnt;
+        ga.cap = sp.cap_s;
+        ga.s_out = s_out;
+        ga.idx_out = idx_out;
+        e = launch_gselect(ga, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        ds->launches += 2;
+        return NEST_OK;
+    }
+
+    CUtensorMap smap;
+    if (!encode_bf16_rows(&smap, ds->K, sp.sample_rows, ds->d, kTcTileKeys, true, sp.stride))
+        return NEST_ERR_CUDA;
+    float* s_s = reinterpret_cast<float*>(scratch + sp.off_s_s);
+    int64_t* i_s = reinterpret_cast<int64_t*>(scratch + sp.off_i_s);
+    // 1. sample pass: every sampled key is a candidate
+    wa.s_sample = nullptr;
+    wa.cand = scratch + sp.off_cand_s;
+    wa.cnt = cnt;
+    wa.cap = sp.cap_s;
+    wa.N = sp.sample_rows;
+    wa.parts = sp.wps.parts;
+    wa.key_stride = sp.stride;
+    e = launch_tc_wide(sp.wps, smap, qmap, wa, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ga.cand = wa.cand;
+    ga.cnt = cnt;
+    ga.cap = sp.cap_s;
+    ga.s_out = s_s;
+    ga.idx_out = i_s;
+    e = launch_gselect(ga, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    // 2. every key, admitted at or below the sample's r-th distance
+    wa.s_sample = s_s;
+    wa.cand = scratch + sp.off_cand_m;
+    wa.cnt = cnt + B;
+    wa.cap = sp.cap_m;
+    wa.N = ds->N;
+    wa.parts = sp.wpm.parts;
+    wa.key_stride = 1;
+    if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+    e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+    ga.cand = wa.cand;
+    ga.cnt = cnt + B;
+    ga.cap = sp.cap_m;
+    ga.s_out = s_out;
+    ga.idx_out = idx_out;
+    e = launch_gselect(ga, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ds->launches += 4;
+    return NEST_OK;
+}
+
 // Plan, check the scratch, launch the scan and the merge tree.  The scratch
 // (64-bit words) is the handle's own or the caller's; timing events are
 // recorded around the scan when `timed`.
@@ -262,6 +397,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
     uint64_t* regionB = scratch + sp.cand_words;
 
     cudaError_t e;
+    if (sp.wide) return launch_wide(ds, sp, q, B, r, s_out, idx_out, scratch, timed, stream);
     if (sp.tc) {
         CUtensorMap qmap;
         if (!encode_bf16_rows(&qmap, q, B, ds->d, 16, false)) return NEST_ERR_CUDA;
@@ -279,6 +415,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         ta.parts = sp.tcp.parts;
         ta.stages = sp.tcp.stages;
         ta.kchunks = (ds->d + 63) / 64;
+        ta.key_stride = 1;
         if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
         e = launch_tc_scan(sp.tcp, ds->keys_map, qmap, ta, stream);
     } else {

@@ -95,13 +95,58 @@ struct TcScanArgs {
     int32_t cap;
     int32_t parts;
     int32_t stages;
-    int32_t kchunks;  // ceil(d / 64)
+    int32_t kchunks;     // ceil(d / 64)
+    int64_t key_stride;  // the tensor map's row i is key i * key_stride (1, or a sample stride)
 };
 
 int tc_cap(int r);
 bool tc_plan_smem(int nq, int r, size_t smem_limit, TcPlan* plan);
 cudaError_t launch_tc_scan(const TcPlan& plan, const CUtensorMap& keys, const CUtensorMap& queries,
                            const TcScanArgs& args, cudaStream_t stream);
+
+// ---------------------------------------------------------------- tc_wide.cu
+// Large query batches: threshold-admission scan into global lists + exact selection.
+struct WidePlan {
+    int nm;       // MMA N = queries per CTA (16, 32, 64, 128 or 256)
+    int stages;
+    int groups;   // query groups of nm
+    int parts;    // key-range parts (whole 128-key tiles)
+    size_t smem;
+};
+
+struct WideArgs {
+    const float* knorm;
+    const void* q;
+    int* status;
+    const float* s_sample;  // B x r sample neighbours (threshold = s[r-1]); null: admit all
+    int32_t r;
+    uint64_t* cand;  // [B][cap] candidate words
+    int32_t* cnt;    // [B] candidates appended (must start at 0)
+    int64_t cap;
+    int64_t N;       // rows of the key tensor map
+    int32_t d;
+    int32_t B;
+    int32_t groups;
+    int32_t parts;
+    int32_t stages;
+    int32_t kchunks;
+    int64_t key_stride;  // row i of the key tensor map is key i * key_stride
+};
+
+struct GselectArgs {
+    uint64_t* cand;  // [B][cap]; reordered in place
+    const int32_t* cnt;
+    int64_t cap;
+    int32_t r;
+    int32_t B;
+    float* s_out;      // B x r
+    int64_t* idx_out;  // B x r
+};
+
+bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* plan);
+cudaError_t launch_tc_wide(const WidePlan& plan, const CUtensorMap& keys,
+                           const CUtensorMap& queries, const WideArgs& args, cudaStream_t stream);
+cudaError_t launch_gselect(const GselectArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- merge.cu
 // Merge candidate lists of each query into its top r.

@@ -223,12 +223,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             qn[b] = (sh.qn_part[0][b] + sh.qn_part[1][b]) + (sh.qn_part[2][b] + sh.qn_part[3][b]);
 
         const int row_in_tile = 32 * quarter + lane;
-        float kn_next = (ntiles > 0 && lo + row_in_tile < hi) ? __ldg(a.knorm + lo + row_in_tile) : 0.f;
+        const int64_t ks = a.key_stride;  // row i of the tensor map is key i * ks
+        float kn_next =
+            (ntiles > 0 && lo + row_in_tile < hi) ? __ldg(a.knorm + (lo + row_in_tile) * ks) : 0.f;
         for (int j = 0; j < ntiles; ++j) {
             const int buf = j & 1;
             const int64_t row = lo + (int64_t)j * kTileM + row_in_tile;
             const float kn = kn_next;
-            kn_next = (row + kTileM < hi) ? __ldg(a.knorm + row + kTileM) : 0.f;
+            kn_next = (row + kTileM < hi) ? __ldg(a.knorm + (row + kTileM) * ks) : 0.f;
             wait_or_abort_tc(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
             tc_fence_after();
             uint32_t acc[16];
@@ -240,7 +242,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int b = 0; b < NQ; ++b) {
                 float dist = fmaf(-2.f, __uint_as_float(acc[b]), qn[b] + kn);
                 dist = (dist <= 0.f) ? 0.f : dist;  // NaN stays NaN and sorts last
-                const uint64_t key = ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)row;
+                const uint64_t key = ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)(row * ks);
                 const bool accept = valid && (b < nqv) && (key <= sh.thr[b]);
                 const uint32_t bal = __ballot_sync(~0u, accept);
                 if (bal) {

@@ -1,0 +1,410 @@
+// tc_wide.cu -- the search for large query batches (Sec. 2.2 / App. A: the
+// r nearest keys of each query, s = -||q - k||^2), where per-query candidate
+// lists no longer fit in one CTA's shared memory.
+//
+//   1. A sampling pre-pass: the same kernel over a tensor map that reads
+//      every stride-th key, admitting every sampled key, and gselect_kernel
+//      on those lists give each query the r-th distance among the sample.
+//      It is an upper bound of the query's true r-th distance, so every key
+//      at or below it is a safe candidate (admission threshold).
+//   2. tc_wide_kernel streams every key tile once per group of up to 256
+//      queries: tcgen05.mma with M = 128 keys, N = up to 256 queries,
+//      K = 16, two TMEM accumulators of N columns; the epilogue warps form
+//      ||q||^2 + ||k||^2 - 2 q.k and append the keys under each query's
+//      threshold to that query's global list (one atomic per warp and query).
+//   3. gselect_kernel takes the exact r smallest of each list (radix select
+//      in place in global memory), sorts them and writes s and idx.
+#include <cmath>
+#include <cuda.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "select.cuh"
+
+namespace nest {
+namespace {
+
+constexpr int kTileM = 128;
+constexpr int kChunkK = 64;
+constexpr int kABytes = kTileM * kChunkK * 2;
+constexpr int kMaxStagesW = 12;
+constexpr int kEpiThreads = 128;
+constexpr int kSelThreads = 1024;
+
+template <int NM>
+struct WideShared {
+    uint64_t full[kMaxStagesW];
+    uint64_t empty[kMaxStagesW];
+    uint64_t acc_full[2];
+    uint64_t acc_empty[2];
+    uint64_t drain;
+    uint64_t thr[NM];
+    float qn[NM];
+    uint32_t tmem_base;
+    int abort;
+    int issued;
+};
+
+template <int NM>
+constexpr int stage_bytes() { return kABytes + NM * kChunkK * 2; }
+
+template <int NM>
+constexpr uint32_t tmem_cols()
+{
+    return (2 * NM) <= 32 ? 32u : (2 * NM) <= 64 ? 64u : (2 * NM) <= 128 ? 128u : (2 * NM) <= 256 ? 256u : 512u;
+}
+
+__device__ __forceinline__ void wait_or_abort_w(uint64_t* bar, uint32_t parity, int* abort_flag,
+                                                int* status)
+{
+    if (*reinterpret_cast<volatile int*>(abort_flag)) return;
+    if (!mbar_wait_bounded(bar, parity)) {
+        record_status(status, NEST_ERR_TIMEOUT);
+        *reinterpret_cast<volatile int*>(abort_flag) = 1;
+    }
+}
+
+template <int NM>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_wide_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
+                   const WideArgs a)
+{
+    constexpr int kStage = stage_bytes<NM>();
+    constexpr uint32_t kCols = tmem_cols<NM>();
+    static_assert(NM % 16 == 0 && NM >= 16 && NM <= 256, "MMA N for M = 128");
+    static_assert(kStage % 1024 == 0, "stage must keep 1024-byte alignment");
+
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    unsigned char* stages = smem;
+    WideShared<NM>& sh = *reinterpret_cast<WideShared<NM>*>(smem + (size_t)a.stages * kStage);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // CTAs of the same key range but different query groups are adjacent, so
+    // they stream the same tiles at about the same time and share them in L2.
+    const int part = blockIdx.x / a.groups, group = blockIdx.x - part * a.groups;
+    const int q0 = group * NM;
+    const int nqv = min(NM, a.B - q0);
+
+    const int64_t tiles = (a.N + kTileM - 1) / kTileM;
+    const int64_t t0 = tiles * part / a.parts, t1 = tiles * (part + 1) / a.parts;
+    const int64_t lo = t0 * kTileM;
+    const int64_t hi = min(a.N, t1 * kTileM);
+    const int ntiles = (int)(t1 - t0);
+    const int kc = a.kchunks;
+    const int nsteps = ntiles * kc;
+
+    if (tid == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&sh.full[s], 1);
+            mbar_init(&sh.empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&sh.acc_full[b], 1);
+            mbar_init(&sh.acc_empty[b], kEpiThreads);
+        }
+        mbar_init(&sh.drain, 1);
+        sh.abort = 0;
+        sh.issued = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) tmem_alloc(&sh.tmem_base, kCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0 && nsteps > 0) {
+            const uint64_t policy = l2_policy_evict_first();
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int s = 0; s < nsteps; ++s) {
+                const int t = s / kc, c = s - t * kc;
+                if (s >= a.stages) {
+                    wait_or_abort_w(&sh.empty[slot], phase ^ 1u, &sh.abort, a.status);
+                    if (*reinterpret_cast<volatile int*>(&sh.abort)) break;
+                }
+                unsigned char* st = stages + (size_t)slot * kStage;
+                mbar_arrive_expect_tx(&sh.full[slot], kStage);
+                // the last query group reads the keys last: let them leave L2 then
+                if (group == a.groups - 1)
+                    tma_load_2d_hint(st, &tmK, c * kChunkK, (int32_t)(lo + (int64_t)t * kTileM),
+                                     &sh.full[slot], policy);
+                else
+                    tma_load_2d(st, &tmK, c * kChunkK, (int32_t)(lo + (int64_t)t * kTileM),
+                                &sh.full[slot]);
+                tma_load_2d(st + kABytes, &tmQ, c * kChunkK, q0, &sh.full[slot]);
+                *reinterpret_cast<volatile int*>(&sh.issued) = s + 1;
+                if (++slot == a.stages) {
+                    slot = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && nsteps > 0) {
+            constexpr uint32_t idesc = mma_idesc_bf16(kTileM, NM);
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int j = 0; j < ntiles; ++j) {
+                const int buf = j & 1;
+                if (j >= 2)
+                    wait_or_abort_w(&sh.acc_empty[buf], (uint32_t)((j >> 1) - 1) & 1u, &sh.abort,
+                                    a.status);
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * NM);
+                for (int c = 0; c < kc; ++c) {
+                    wait_or_abort_w(&sh.full[slot], phase, &sh.abort, a.status);
+                    tc_fence_after();
+                    const unsigned char* st = stages + (size_t)slot * kStage;
+                    const uint64_t ad = smem_desc_sw128(st);
+                    const uint64_t bd = smem_desc_sw128(st + kABytes);
+#pragma unroll
+                    for (int k = 0; k < kChunkK / 16; ++k)
+                        mma_bf16(d_tmem, ad + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
+                    mma_commit(&sh.empty[slot]);
+                    if (++slot == a.stages) {
+                        slot = 0;
+                        phase ^= 1u;
+                    }
+                }
+                mma_commit(&sh.acc_full[buf]);
+            }
+            mma_commit(&sh.drain);
+            (void)mbar_wait_bounded(&sh.drain, 0);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int e = tid - 64;
+        const int quarter = warp & 3;
+        // Admission threshold of each query: every key at or below the r-th
+        // distance of the sample (an upper bound of the true r-th distance),
+        // or every key on the sampling pass itself (no s_sample).
+        for (int j = e; j < NM; j += kEpiThreads) {
+            uint64_t thr = kNoCandidate;
+            if (a.s_sample != nullptr && j < nqv) {
+                const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                if (s_r > -INFINITY)
+                    thr = ((uint64_t)__float_as_uint(-s_r) << 32) | 0xFFFFFFFFull;
+            }
+            sh.thr[j] = thr;
+        }
+        // ||q||^2 of the group's queries (warp w: queries w, w + 4, ...), bf16 values
+        const unsigned char* qb = static_cast<const unsigned char*>(a.q);
+        const int chunks = a.d / 8;  // 16-byte chunks of a row (d * 2 is a multiple of 16)
+        for (int j = warp - 2; j < NM; j += 4) {
+            float s = 0.f;
+            if (j < nqv) {
+                const unsigned char* row = qb + (size_t)(q0 + j) * a.d * 2;
+                for (int c = lane; c < chunks; c += 32) {
+                    const uint4 v = ld_global_nc_v4(row + (size_t)c * 16);
+                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float lo = __uint_as_float(w[i] << 16);
+                        const float hi = __uint_as_float(w[i] & 0xffff0000u);
+                        s = fmaf(lo, lo, s);
+                        s = fmaf(hi, hi, s);
+                    }
+                }
+            }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
+            if (lane == 0) sh.qn[j] = s;
+        }
+        named_barrier(2, kEpiThreads);
+
+        const int row_in_tile = 32 * quarter + lane;
+        const int64_t ks = a.key_stride;  // row i of the tensor map is key i * ks
+        float kn_next =
+            (ntiles > 0 && lo + row_in_tile < hi) ? __ldg(a.knorm + (lo + row_in_tile) * ks) : 0.f;
+        for (int j = 0; j < ntiles; ++j) {
+            const int buf = j & 1;
+            const int64_t row = lo + (int64_t)j * kTileM + row_in_tile;
+            const float kn = kn_next;
+            kn_next = (row + kTileM < hi) ? __ldg(a.knorm + (row + kTileM) * ks) : 0.f;
+            const bool valid = row < hi;
+            wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
+            tc_fence_after();
+            const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);
+#pragma unroll 1
+            for (int c0 = 0; c0 < NM; c0 += 16) {
+                uint32_t acc[16];
+                tmem_ld_16(tbase + (uint32_t)c0, acc);
+                if (c0 + 16 == NM) {  // the whole accumulator has been read
+                    tc_fence_before();
+                    mbar_arrive(&sh.acc_empty[buf]);
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int col = c0 + i;
+                    float dist = fmaf(-2.f, __uint_as_float(acc[i]), sh.qn[col] + kn);
+                    dist = (dist <= 0.f) ? 0.f : dist;
+                    const uint64_t key =
+                        ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)(row * ks);
+                    // padding columns (no query) never append
+                    const bool accept = valid && col < nqv && key <= sh.thr[col];
+                    const uint32_t bal = __ballot_sync(~0u, accept);
+                    if (bal) {
+                        const int leader = __ffs(bal) - 1;
+                        long long at = 0;
+                        if (lane == leader) at = atomicAdd(&a.cnt[q0 + col], __popc(bal));
+                        at = __shfl_sync(~0u, at, leader);
+                        if (accept) {
+                            const long long pos = at + __popc(bal & lanemask_lt());
+                            if (pos < a.cap) a.cand[(int64_t)(q0 + col) * a.cap + pos] = key;
+                            else record_status(a.status, NEST_ERR_OVERFLOW);
+                        }
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kCols);
+    }
+    if (tid == 0 && *reinterpret_cast<volatile int*>(&sh.abort)) {
+        const int issued = *reinterpret_cast<volatile int*>(&sh.issued);
+        for (int s = max(0, issued - a.stages); s < issued; ++s)
+            (void)mbar_wait_bounded(&sh.full[s % a.stages], (uint32_t)(s / a.stages) & 1u);
+    }
+}
+
+// ---------------------------------------------------------------- exact top-r of each global list
+struct GselShared {
+    int cnt;
+    uint64_t thr;
+    SelectSmem<kSelThreads, 1> sel;
+};
+
+__global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectArgs a)
+{
+    extern __shared__ __align__(16) uint64_t sort_buf[];  // next_pow2(r) words
+    __shared__ GselShared sh;
+    const int tid = threadIdx.x;
+    const int q = blockIdx.x;
+    uint64_t* list = a.cand + (int64_t)q * a.cap;
+    if (tid == 0) {
+        const int c = a.cnt[q];
+        sh.cnt = c < a.cap ? c : (int)a.cap;
+        sh.thr = kNoCandidate;
+    }
+    __syncthreads();
+    // keeps the r smallest at the front of the list, in place
+    select_smallest<kSelThreads, 1>(list, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
+                                    [] { __syncthreads(); });
+    const int n = sh.cnt;
+    int P2 = 1;
+    while (P2 < (n > 0 ? n : 1)) P2 <<= 1;
+    for (int j = tid; j < P2; j += kSelThreads) sort_buf[j] = j < n ? list[j] : kNoCandidate;
+    __syncthreads();
+    for (int k = 2; k <= P2; k <<= 1) {
+        for (int jj = k >> 1; jj > 0; jj >>= 1) {
+            for (int i = tid; i < P2; i += kSelThreads) {
+                const int l = i ^ jj;
+                if (l > i) {
+                    const uint64_t x = sort_buf[i], y = sort_buf[l];
+                    if ((x > y) == ((i & k) == 0)) {
+                        sort_buf[i] = y;
+                        sort_buf[l] = x;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+    float* so = a.s_out + (int64_t)q * a.r;
+    int64_t* io = a.idx_out + (int64_t)q * a.r;
+    for (int j = tid; j < a.r; j += kSelThreads) {
+        if (j < n) {
+            const uint64_t e = sort_buf[j];
+            so[j] = -__uint_as_float((uint32_t)(e >> 32));
+            io[j] = (int64_t)(uint32_t)e;
+        } else {
+            so[j] = -INFINITY;
+            io[j] = -1;
+        }
+    }
+}
+
+template <int NM>
+size_t wide_fixed()
+{
+    return 1024 + sizeof(WideShared<NM>);
+}
+
+template <int NM>
+bool wide_plan_nm(size_t smem_limit, WidePlan* p)
+{
+    const size_t fixed = wide_fixed<NM>();
+    const size_t st = (size_t)stage_bytes<NM>();
+    if (fixed + 3 * st > smem_limit) return false;
+    int stages = (int)((smem_limit - fixed) / st);
+    stages = stages > kMaxStagesW ? kMaxStagesW : stages;
+    p->nm = NM;
+    p->stages = stages;
+    p->smem = fixed + (size_t)stages * st;
+    return true;
+}
+
+template <int NM>
+cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
+                           const WideArgs& a, cudaStream_t stream)
+{
+    auto kern = tc_wide_kernel<NM>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    if (e != cudaSuccess) return e;
+    kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* p)
+{
+    switch (nm) {
+    case 16: return wide_plan_nm<16>(smem_limit, p);
+    case 32: return wide_plan_nm<32>(smem_limit, p);
+    case 64: return wide_plan_nm<64>(smem_limit, p);
+    case 128: return wide_plan_nm<128>(smem_limit, p);
+    case 256: return wide_plan_nm<256>(smem_limit, p);
+    default: return false;
+    }
+}
+
+cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
+                           const WideArgs& a, cudaStream_t stream)
+{
+    switch (p.nm) {
+    case 16: return wide_launch_nm<16>(p, tmK, tmQ, a, stream);
+    case 32: return wide_launch_nm<32>(p, tmK, tmQ, a, stream);
+    case 64: return wide_launch_nm<64>(p, tmK, tmQ, a, stream);
+    case 128: return wide_launch_nm<128>(p, tmK, tmQ, a, stream);
+    case 256: return wide_launch_nm<256>(p, tmK, tmQ, a, stream);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_gselect(const GselectArgs& a, cudaStream_t stream)
+{
+    int P2 = 1;
+    while (P2 < a.r) P2 <<= 1;
+    const size_t smem = (size_t)P2 * sizeof(uint64_t);
+    cudaError_t e = cudaFuncSetAttribute(gselect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    gselect_kernel<<<a.B, kSelThreads, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace nest

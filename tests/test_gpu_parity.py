@@ -38,7 +38,12 @@ def _cand_counts(B, N, seg_off):
 
 
 def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, exact=False,
-                  oracle_threads=None):
+                  oracle_threads=None, check_rows=None):
+    """GPU step through the C ABI, then the oracle on the same bytes.
+
+    ``check_rows`` restricts the oracle (and the comparison) to those query
+    rows of a full-scan batch; the GPU always runs the whole batch.
+    """
     dev = torch.device("cuda")
     K, V, q, p_lm = K.to(dev), V.to(dev), q.to(dev), p_lm.to(dev)
     so = seg_off.to(dev) if seg_off is not None else None
@@ -46,18 +51,21 @@ def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, e
     out = ds.step(q, r, p_lm, mu, lam, seg_off=so, want_p_knn=True)
     torch.cuda.synchronize()
     assert ds.device_status() == 0
-    s_g = out["s"].cpu().numpy()
-    i_g = out["idx"].cpu().numpy()
-    K_np, q_np, V_np = _np(K), _np(q), V.cpu().numpy()
-    p_lm_np = p_lm.cpu().numpy()
+    rows_sel = slice(None) if check_rows is None else list(check_rows)
+    s_g = out["s"].cpu().numpy()[rows_sel]
+    i_g = out["idx"].cpu().numpy()[rows_sel]
+    K_np, V_np = _np(K), V.cpu().numpy()
+    q_np = _np(q)[rows_sel]
+    p_lm_np = p_lm.cpu().numpy()[rows_sel]
     so_np = seg_off.cpu().numpy() if seg_off is not None else None
     ref = oracle.knn_step(K_np, V_np, q_np, r, p_lm_np, mu, lam, vocab, seg_off=so_np,
                           nthreads=oracle_threads)
     rows = check_search(s_g, i_g, ref["s"], ref["idx"], K_np, q_np, dtype,
-                        _cand_counts(q.shape[0], K.shape[0], seg_off), exact=exact)
-    check_mix(out["p_m"].cpu().numpy(), s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
-              p_knn_gpu=out["p_knn"].cpu().numpy())
-    check_mix_end_to_end(out["p_m"].cpu().numpy(), ref["p_m"], rows)
+                        _cand_counts(q_np.shape[0], K.shape[0], seg_off), exact=exact)
+    p_m = out["p_m"].cpu().numpy()[rows_sel]
+    check_mix(p_m, s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
+              p_knn_gpu=out["p_knn"].cpu().numpy()[rows_sel])
+    check_mix_end_to_end(p_m, ref["p_m"], rows)
     ds.close()
     return out, ref, rows
 
@@ -289,3 +297,29 @@ def test_step_host_matches_device_step(nest):
     assert torch.equal(host["p_m"], o["p_m"].cpu())
     assert torch.equal(host["idx"], o["idx"].cpu())
     ds.close()
+
+
+# ---------------------------------------------------------------- large query batches
+
+def test_wide_batch_with_sampled_thresholds(nest):
+    """B=40 queries (more than one CTA keeps lists for at r=256): sample pass,
+    thresholded pass, exact selection of the survivors."""
+    K, V, q, p_lm = _random_case(200000, 256, 40, 700, "bf16", seed=21, centres=64)
+    run_and_check(nest, K, V, q, p_lm, 256, 1 / 16, 0.8, 700, "bf16")
+
+
+def test_wide_batch_single_pass_over_300_queries(nest):
+    """B=300 > 256 (two query groups); the datastore is small enough that the
+    sample is every key."""
+    K, V, q, p_lm = _random_case(100003, 128, 300, 500, "bf16", seed=22, centres=32)
+    run_and_check(nest, K, V, q, p_lm, 64, 1 / np.sqrt(128), 0.8, 500, "bf16")
+
+
+def test_large_batch_shape_sampled_rows(nest):
+    """Large-batch shape: bf16 d=4096, B=512, r=256, clustered keys (N reduced
+    to 524,288); the oracle checks 12 query rows spread over the batch."""
+    w = synth.WORKLOADS["large_batch"]
+    x = synth.make_inputs(w, device="cuda", N=1 << 19)
+    rows = list(range(0, 512, 43))
+    run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
+                  check_rows=rows)
