@@ -51,6 +51,9 @@ def parse():
                    help="queries in the oracle's bounded sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=200)
+    p.add_argument("--sweep", default=None,
+                   help="comma-separated query batch sizes measured on one datastore, one JSON "
+                        "line each (e.g. 1,8,64,256 for the d=8192 workload)")
     return p.parse_args()
 
 
@@ -308,9 +311,25 @@ def main():
     nest_build.build()
 
     dev = torch.device("cuda", local)
-    x = synth.make_inputs(w, device=dev, B=args.B, N=args.N, seed=w.seed + rank)
-    B = x.q.shape[0]
+    sweep = [int(v) for v in args.sweep.split(",")] if args.sweep else [args.B]
+    B_gen = max(b for b in sweep if b is not None) if any(b is not None for b in sweep) else None
+    x = synth.make_inputs(w, device=dev, B=B_gen, N=args.N, seed=w.seed + rank)
     ds = nest.Datastore(x.K, x.V, w.vocab)
+    for B in sweep:
+        line = measure(args, w, x, ds, B if B is not None else x.q.shape[0], world, rank, local)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+    ds.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def measure(args, w, x_all, ds, B, world, rank, local):
+    """Time one batch size on an existing datastore; returns the JSON line (rank 0)."""
+    x = synth.Inputs(K=x_all.K, V=x_all.V, q=x_all.q[:B].contiguous(),
+                     p_lm=x_all.p_lm[:B].contiguous(),
+                     seg_off=x_all.seg_off[:B + 1].contiguous() if x_all.seg_off is not None else None)
     out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off)  # allocates scratch once
     stream = torch.cuda.current_stream()
     for _ in range(max(3, args.warmup)):
@@ -359,8 +378,7 @@ def main():
     hbm_peak, tc_peak, peak_kind = peaks()
     t_hbm = alg_bytes / (hbm_peak * 1e9)
     t_tc = alg_flops / (tc_peak * 1e12)
-    wide = w.dtype == "bf16" and x.seg_off is None and B > 16
-    kernel = ("tc_wide_kernel" if wide else "tc_scan_kernel") if w.dtype == "bf16" else "scan_topr_kernel"
+    kernel = ds.search_path(B, w.r, ragged=x.seg_off is not None)
     if t_tc > t_hbm:
         achieved = alg_flops / (scan_avg_ms / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s",
@@ -401,6 +419,7 @@ def main():
         cpu = cpu_baseline(w, x, min(args.oracle_queries, B))
         cpu.pop("seconds", None)
 
+    line = None
     if rank == 0:
         line = {
             "metric": "queries/s for fused kNN search+top-r+p_M mix", "value": value,
@@ -412,11 +431,7 @@ def main():
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clk,
         }
-        print(json.dumps(line), flush=True)
-    ds.close()
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+    return line
 
 
 if __name__ == "__main__":

@@ -224,6 +224,17 @@ NEST_API nest_status_t nest_device_status(nest_datastore_t* ds, void* stream);
 NEST_API nest_status_t nest_timing_enable(nest_datastore_t* ds, int32_t on);
 NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, int64_t* launches);
 
+/*
+ * Which distance scan a search of this shape runs on this datastore:
+ *   0  CUDA-core scan with per-CTA top-r (fp32 keys, or rows TMA cannot map)
+ *   1  tensor-core scan with per-CTA top-r (bf16 keys, query groups of <= 16)
+ *   2  tensor-core scan of large query batches against sampled admission
+ *      thresholds (bf16 keys, more queries than one CTA keeps lists for)
+ * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
+ */
+NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,
+                                  int32_t ragged);
+
 /* Kernels this handle has launched since it was created (all kinds). */
 NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
 

@@ -695,6 +695,15 @@ nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, int64_t* 
 
 int64_t nest_launch_count(const nest_datastore_t* ds) { return ds ? ds->launches : 0; }
 
+int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r, int32_t ragged)
+{
+    if (!ds || B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R) return -(int32_t)NEST_ERR_INVALID_ARG;
+    SearchPlan sp;
+    const nest_status_t st = plan_search(ds, B, r, ragged != 0, &sp);
+    if (st != NEST_OK) return -(int32_t)st;
+    return sp.wide ? 2 : (sp.tc ? 1 : 0);
+}
+
 const char* nest_status_string(nest_status_t s)
 {
     switch (s) {

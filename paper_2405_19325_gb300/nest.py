@@ -43,6 +43,7 @@ SIGNATURES = {
     "nest_timing_read": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_double),
                                         ctypes.POINTER(_I64)]),
     "nest_launch_count": (_I64, [_P]),
+    "nest_search_path": (_I32, [_P, _I32, _I32, _I32]),
     "nest_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "nest_version": (_I32, []),
 }
@@ -279,6 +280,15 @@ class Datastore:
 
     def launch_count(self) -> int:
         return int(self._lib.nest_launch_count(self._h))
+
+    SEARCH_PATHS = {0: "scan_topr_kernel", 1: "tc_scan_kernel", 2: "tc_wide_kernel"}
+
+    def search_path(self, B: int, r: int, ragged: bool = False) -> str:
+        """Name of the distance-scan kernel a search of this shape runs."""
+        code = int(self._lib.nest_search_path(self._h, B, r, int(ragged)))
+        if code < 0:
+            raise NestError(-code, "nest_search_path")
+        return self.SEARCH_PATHS[code]
 
     def _check_rows(self, p_lm: torch.Tensor, B: int) -> None:
         if p_lm.dim() != 2 or p_lm.shape[0] != B or p_lm.shape[1] != self.vocab:

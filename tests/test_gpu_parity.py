@@ -305,6 +305,10 @@ def test_wide_batch_with_sampled_thresholds(nest):
     """B=40 queries (more than one CTA keeps lists for at r=256): sample pass,
     thresholded pass, exact selection of the survivors."""
     K, V, q, p_lm = _random_case(200000, 256, 40, 700, "bf16", seed=21, centres=64)
+    ds = nest.Datastore(K.cuda(), V.cuda(), 700)
+    assert ds.search_path(40, 256) == "tc_wide_kernel"
+    assert ds.search_path(4, 256) == "tc_scan_kernel"
+    ds.close()
     run_and_check(nest, K, V, q, p_lm, 256, 1 / 16, 0.8, 700, "bf16")
 
 
@@ -323,3 +327,69 @@ def test_large_batch_shape_sampled_rows(nest):
     rows = list(range(0, 512, 43))
     run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
                   check_rows=rows)
+
+
+# ---------------------------------------------------------------- full-size, sampled rows
+
+def _chunks(K, rows=65536):
+    for lo in range(0, K.shape[0], rows):
+        yield lo, synth.to_numpy_raw(K[lo:min(K.shape[0], lo + rows)])
+
+
+def test_large_batch_full_size_sampled_rows(nest):
+    """bf16 d=4096, N=4,194,304, B=512, r=256 (the benchmarked large-batch launch):
+    the oracle checks query rows 0 and 511 over all keys."""
+    w = synth.WORKLOADS["large_batch"]
+    x = synth.make_inputs(w, device="cuda")
+    ds = nest.Datastore(x.K, x.V, w.vocab)
+    out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam)
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    s_all, i_all = out["s"].cpu().numpy(), out["idx"].cpu().numpy()
+    qidx = [0, 511]
+    _check_rows_full_size_simple(out, x.K, x.V, x.q, qidx, x.p_lm, w, s_all, i_all)
+    ds.close()
+
+
+def _check_rows_full_size_simple(out, K, V, q, qidx, p_lm, w, s_all, i_all):
+    q_np = synth.to_numpy_raw(q[qidx])
+    s_or, i_or = oracle.knn_search_chunked(_chunks(K), q_np, w.r)
+    V_np = V.cpu().numpy()
+    for j, b in enumerate(qidx):
+        i_g = i_all[b]
+        # exact distances of the union of both lists, from the rows themselves
+        union = np.unique(np.concatenate([i_g, i_or[j]]))
+        K_rows = synth.to_numpy_raw(K[torch.as_tensor(union, device=K.device)])
+        where = {int(k): n for n, k in enumerate(union)}
+        g_loc = np.array([where[int(k)] for k in i_g])[None]
+        o_loc = np.array([where[int(k)] for k in i_or[j]])[None]
+        rows = check_search(s_all[b:b + 1], g_loc, s_or[j:j + 1], o_loc, K_rows, q_np[j:j + 1],
+                            w.dtype, np.array([K.shape[0]]))
+        check_mix(out["p_m"][b:b + 1].cpu().numpy(), s_all[b:b + 1], i_all[b:b + 1], V_np,
+                  p_lm[b:b + 1].cpu().numpy(), w.mu, w.lam, w.vocab)
+        if rows:
+            P, n = oracle.pknn(s_or[j:j + 1], i_or[j:j + 1], V_np, w.mu, w.vocab)
+            ref = oracle.mix(p_lm[b:b + 1].cpu().numpy(), P, w.lam, n)
+            check_mix_end_to_end(out["p_m"][b:b + 1].cpu().numpy(), ref, [0])
+
+
+def test_hidden8192_full_size_B_sweep(nest):
+    """bf16 d=8192, N=8,388,608 clustered keys (128 GiB), r=1024, B in {1, 8, 64, 256}:
+    four kernel paths on one datastore.  Query 0 must get the same neighbours on
+    every path; the oracle checks queries 0 and 255 over all keys."""
+    w = synth.WORKLOADS["hidden8192"]
+    x = synth.make_inputs(w, device="cuda", B=256)
+    ds = nest.Datastore(x.K, x.V, w.vocab)
+    first = None
+    for B in (1, 8, 64, 256):
+        out = ds.step(x.q[:B].contiguous(), w.r, x.p_lm[:B].contiguous(), w.mu, w.lam)
+        torch.cuda.synchronize()
+        assert ds.device_status() == 0, f"B={B}"
+        i0 = out["idx"][0].cpu().numpy()
+        if first is None:
+            first = i0
+        else:
+            assert set(first.tolist()) == set(i0.tolist()), f"B={B}: query 0 differs from B=1"
+    s_all, i_all = out["s"].cpu().numpy(), out["idx"].cpu().numpy()
+    _check_rows_full_size_simple(out, x.K, x.V, x.q, [0, 255], x.p_lm, w, s_all, i_all)
+    ds.close()
