@@ -19,6 +19,12 @@ Functions and the passages they restate:
 * ``pknn``     -- Eq. 2
 * ``mix``      -- Eq. 3
 * ``rrc``      -- Eq. 4
+* ``decide``   -- greedy token and span start (Eq. 5), span decision (Eq. 6)
+* ``verify``   -- relaxed speculative decoding of drafted spans (Eq. 7)
+
+``knn_search`` also takes ``exclude`` (a boolean per key): excluded keys are
+left out of the candidate set, as accepted spans are masked out of the
+datastore for the rest of a generation (Sec. 3.4).
 """
 from __future__ import annotations
 
@@ -70,6 +76,13 @@ def _load():
         lib.nest_oracle_mix.restype = ctypes.c_int
         lib.nest_oracle_rrc.argtypes = [P, P, ctypes.c_int32, ctypes.c_double, ctypes.c_double]
         lib.nest_oracle_rrc.restype = ctypes.c_double
+        lib.nest_oracle_decide.argtypes = [P, ctypes.c_int32, P, P, P, ctypes.c_int64,
+                                           ctypes.c_int32, ctypes.c_double, ctypes.c_double,
+                                           P, P, P, P]
+        lib.nest_oracle_decide.restype = ctypes.c_int
+        lib.nest_oracle_verify.argtypes = [P, ctypes.c_int32, P, ctypes.c_int32, P, ctypes.c_int32,
+                                           ctypes.c_double, P, P, P]
+        lib.nest_oracle_verify.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -125,29 +138,38 @@ def topr(D: np.ndarray, idx: np.ndarray, r: int) -> tuple[np.ndarray, np.ndarray
 
 
 def knn_search(K: np.ndarray, q: np.ndarray, r: int, seg_off: np.ndarray | None = None,
-               nthreads: int | None = None) -> tuple[np.ndarray, np.ndarray]:
+               nthreads: int | None = None,
+               exclude: np.ndarray | None = None) -> tuple[np.ndarray, np.ndarray]:
     """Top-r search of every query.
 
     Returns (s, idx), each B x r: s = -||q - k||^2 in fp64, nearest first
     (ties to the smaller key index), padded with s = -inf, idx = -1.  With
     ``seg_off`` (B + 1 offsets) query b searches only keys
-    [seg_off[b], seg_off[b+1]) and idx stays a global key index.
+    [seg_off[b], seg_off[b+1]) and idx stays a global key index.  Keys with
+    ``exclude[i]`` true are not candidates.
     """
     B = q.shape[0]
     s = np.empty((B, r), dtype=np.float64)
     I = np.empty((B, r), dtype=np.int64)
+    keep_all = None if exclude is None else ~np.asarray(exclude, dtype=bool)
     if seg_off is None:
         D = sqdist(K, q, nthreads)
         allidx = np.arange(K.shape[0], dtype=np.int64)
         for b in range(B):
-            Db, Ib, _ = topr(D[b], allidx, r)
+            Db, Ib = D[b], allidx
+            if keep_all is not None:
+                Db, Ib = Db[keep_all], Ib[keep_all]
+            Db, Ib, _ = topr(Db, Ib, r)
             s[b], I[b] = -Db, Ib
     else:
         seg_off = np.asarray(seg_off, dtype=np.int64)
         for b in range(B):
             lo, hi = int(seg_off[b]), int(seg_off[b + 1])
             D = sqdist(K[lo:hi], q[b:b + 1], nthreads)[0]
-            Db, Ib, _ = topr(D, np.arange(lo, hi, dtype=np.int64), r)
+            Ib = np.arange(lo, hi, dtype=np.int64)
+            if keep_all is not None:
+                D, Ib = D[keep_all[lo:hi]], Ib[keep_all[lo:hi]]
+            Db, Ib, _ = topr(D, Ib, r)
             s[b], I[b] = -Db, Ib
     return s, I
 
@@ -217,6 +239,48 @@ def rrc(s: np.ndarray, idx: np.ndarray, alpha: float, tau: float) -> np.ndarray:
     return np.array([lib.nest_oracle_rrc(_ptr(s[b]), _ptr(idx[b]), s.shape[1],
                                          float(alpha), float(tau))
                      for b in range(s.shape[0])], dtype=np.float64)
+
+
+def decide(p_m: np.ndarray, s: np.ndarray, idx: np.ndarray, values: np.ndarray, lam,
+           delta: float):
+    """Eq. 5 / Eq. 6 per row: (token, p_max, span_key, use_span)."""
+    p_m = np.ascontiguousarray(np.atleast_2d(p_m), dtype=np.float64)
+    s = np.ascontiguousarray(np.atleast_2d(s), dtype=np.float64)
+    idx = np.ascontiguousarray(np.atleast_2d(idx), dtype=np.int64)
+    values = np.ascontiguousarray(values, dtype=np.int32)
+    B, V = p_m.shape
+    lams = np.broadcast_to(np.asarray(lam, dtype=np.float64), (B,))
+    tok = np.empty(B, np.int32)
+    pmax = np.empty(B, np.float64)
+    key = np.empty(B, np.int64)
+    use = np.empty(B, np.int32)
+    lib = _load()
+    for b in range(B):
+        t, pm = ctypes.c_int32(), ctypes.c_double()
+        k, u = ctypes.c_int64(), ctypes.c_int32()
+        if lib.nest_oracle_decide(_ptr(p_m[b]), V, _ptr(s[b]), _ptr(idx[b]), _ptr(values),
+                                  values.shape[0], s.shape[1], float(lams[b]), float(delta),
+                                  ctypes.byref(t), ctypes.byref(pm), ctypes.byref(k),
+                                  ctypes.byref(u)) != 0:
+            raise ValueError("nest_oracle_decide rejected its arguments")
+        tok[b], pmax[b], key[b], use[b] = t.value, pm.value, k.value, u.value
+    return tok, pmax, key, use
+
+
+def verify(p_m: np.ndarray, draft: np.ndarray, span_off: np.ndarray, gamma: float):
+    """Eq. 7 over drafted spans: (ratio[rows], accept[rows], n_accept[spans])."""
+    p_m = np.ascontiguousarray(np.atleast_2d(p_m), dtype=np.float64)
+    draft = np.ascontiguousarray(draft, dtype=np.int32)
+    span_off = np.ascontiguousarray(span_off, dtype=np.int32)
+    rows, V = p_m.shape
+    spans = span_off.shape[0] - 1
+    ratio = np.empty(rows, np.float64)
+    acc = np.empty(rows, np.int32)
+    n_acc = np.empty(max(spans, 0), np.int32)
+    if _load().nest_oracle_verify(_ptr(p_m), V, _ptr(draft), rows, _ptr(span_off), spans,
+                                  float(gamma), _ptr(ratio), _ptr(acc), _ptr(n_acc)) != 0:
+        raise ValueError("nest_oracle_verify rejected its arguments")
+    return ratio, acc, n_acc
 
 
 def knn_step(K, values, q, r, p_lm, mu, lam, vocab, seg_off=None, nthreads=None):

@@ -210,3 +210,85 @@ double nest_oracle_rrc(const double* s, const int64_t* idx, int32_t r,
     double ratio = (hi == 0.0) ? 1.0 : lo / hi;
     return 1.0 / (1.0 + exp(-(ratio - alpha) / tau));
 }
+
+/*
+ * Greedy token and span start for one row (Eq. 5 and Eq. 6, Sec. 3.3;
+ * the span-selection steps of Algorithm 1).
+ *
+ *   token    = argmax_w p_m[w]; ties go to the smaller token id.
+ *   span_key = the neighbour whose value is `token` and whose own term
+ *              exp(mu s_i) is largest, i.e. the largest s_i (ties: smaller
+ *              key index); -1 when no neighbour has that value.  Eq. 5 and
+ *              Algorithm 1 write this as an argmax of p_kNN over neighbours
+ *              with value w_t, which is one number for all of them; the
+ *              max-pooling is read as pooling the neighbours' own terms.
+ *   use_span = 1 when lambda <= delta and a span start exists (Eq. 6 emits
+ *              the n-gram continuation), else 0 (emit the token).
+ * p_m has vocab entries; s, idx are the r neighbours (idx < 0: empty slot).
+ * Returns 0, or -1 on a bad argument.
+ */
+int nest_oracle_decide(const double* p_m, int32_t vocab, const double* s, const int64_t* idx,
+                       const int32_t* values, int64_t N, int32_t r, double lambda, double delta,
+                       int32_t* token, double* p_max, int64_t* span_key, int32_t* use_span)
+{
+    if (!p_m || vocab < 1 || !s || !idx || !values || r < 1 || !token || !p_max || !span_key ||
+        !use_span)
+        return -1;
+    int32_t best = 0;
+    for (int32_t w = 1; w < vocab; ++w)
+        if (p_m[w] > p_m[best]) best = w;
+    *token = best;
+    *p_max = p_m[best];
+    int64_t key = -1;
+    double key_s = 0.0;
+    for (int32_t i = 0; i < r; ++i) {
+        if (idx[i] < 0 || idx[i] >= N) continue;
+        if (values[idx[i]] != best) continue;
+        if (key < 0 || s[i] > key_s || (s[i] == key_s && idx[i] < key)) {
+            key = idx[i];
+            key_s = s[i];
+        }
+    }
+    *span_key = key;
+    *use_span = (lambda <= delta && key >= 0) ? 1 : 0;
+    return 0;
+}
+
+/*
+ * Relaxed speculative decoding of drafted spans (Eq. 7, Sec. 3.4; the
+ * verification loop of Algorithm 1).  Row b of p_m (rows x vocab) is p_M at
+ * draft position b and draft[b] the drafted token there; span j covers rows
+ * [span_off[j], span_off[j+1]).
+ *
+ *   ratio[b]    = p_m[b][draft[b]] / (gamma * max_w p_m[b][w])
+ *   accept[b]   = 1 if min(1, ratio[b]) > 1/2, else 0 (Algorithm 1 stops at
+ *                 the first position whose acceptance is at most 1/2)
+ *   n_accept[j] = number of leading accepted positions of span j
+ *
+ * A row whose maximum is 0 has ratio 0.  Returns 0, or -1 on a bad argument.
+ */
+int nest_oracle_verify(const double* p_m, int32_t vocab, const int32_t* draft, int32_t rows,
+                       const int32_t* span_off, int32_t spans, double gamma, double* ratio,
+                       int32_t* accept, int32_t* n_accept)
+{
+    if (!p_m || vocab < 1 || !draft || rows < 0 || !span_off || spans < 0 || !(gamma > 0.0) ||
+        !ratio || !accept || !n_accept)
+        return -1;
+    for (int32_t b = 0; b < rows; ++b) {
+        if (draft[b] < 0 || draft[b] >= vocab) return -1;
+        double mx = 0.0;
+        for (int32_t w = 0; w < vocab; ++w)
+            if (p_m[(int64_t)b * vocab + w] > mx) mx = p_m[(int64_t)b * vocab + w];
+        const double p = p_m[(int64_t)b * vocab + draft[b]];
+        ratio[b] = mx > 0.0 ? p / (gamma * mx) : 0.0;
+        const double a = ratio[b] < 1.0 ? ratio[b] : 1.0;
+        accept[b] = a > 0.5 ? 1 : 0;
+    }
+    for (int32_t j = 0; j < spans; ++j) {
+        if (span_off[j] < 0 || span_off[j + 1] < span_off[j] || span_off[j + 1] > rows) return -1;
+        int32_t n = 0;
+        while (span_off[j] + n < span_off[j + 1] && accept[span_off[j] + n]) ++n;
+        n_accept[j] = n;
+    }
+    return 0;
+}

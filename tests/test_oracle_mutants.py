@@ -24,6 +24,14 @@ MUTANTS = {
     "no_max_subtraction": ("Z += exp(mu * (s[i] - s_max));", "Z += exp(mu * s[i]);"),
     "swapped_lambda": ("(1.0 - lambda) * p_knn[w]", "lambda * p_knn[w]"),
     "rrc_without_abs": ("double a = fabs(s[i]);", "double a = s[i];"),
+    "argmax_ties_to_larger_id": ("if (p_m[w] > p_m[best]) best = w;",
+                                 "if (p_m[w] >= p_m[best]) best = w;"),
+    "span_start_farthest": ("if (key < 0 || s[i] > key_s", "if (key < 0 || s[i] < key_s"),
+    "span_rule_strict": ("*use_span = (lambda <= delta && key >= 0)",
+                         "*use_span = (lambda < delta && key >= 0)"),
+    "verify_without_gamma": ("ratio[b] = mx > 0.0 ? p / (gamma * mx) : 0.0;",
+                             "ratio[b] = mx > 0.0 ? p / mx : 0.0;"),
+    "verify_accepts_half": ("accept[b] = a > 0.5 ? 1 : 0;", "accept[b] = a >= 0.5 ? 1 : 0;"),
 }
 
 

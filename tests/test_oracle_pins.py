@@ -309,3 +309,104 @@ def test_tiny_workload_inputs_are_seeded_and_shaped():
     # Zipf(1.1): token 0 is the most frequent value
     counts = torch.bincount(a.V.long(), minlength=w.vocab)
     assert int(counts.argmax()) == 0
+
+
+# ---------------------------------------------------------------- Eq. 5 / Eq. 6
+
+def _brute_decide(p_m, s, idx, values, lam, delta):
+    token = int(np.argmax(p_m))  # numpy: first maximum = smaller token id
+    cands = sorted((-float(s[i]), int(idx[i])) for i in range(len(idx))
+                   if idx[i] >= 0 and values[idx[i]] == token)
+    key = cands[0][1] if cands else -1
+    return token, float(p_m[token]), key, int(lam <= delta and key >= 0)
+
+
+def test_decide_matches_brute_force_with_ties():
+    rng = np.random.default_rng(30)
+    N, V, r = 300, 12, 40
+    values = rng.integers(0, V, N).astype(np.int32)
+    for trial in range(40):
+        p_m = rng.dirichlet(np.ones(V))
+        if trial % 3 == 0:  # planted tie on the maximum
+            j, k = rng.choice(V, 2, replace=False)
+            p_m[j] = p_m[k] = p_m.max() + 0.01
+        s = -np.round(rng.uniform(0, 5, r), 1)  # rounded: ties in s
+        idx = rng.choice(N, r, replace=False).astype(np.int64)
+        idx[rng.random(r) < 0.1] = -1
+        lam = float(rng.uniform())
+        got = oracle.decide(p_m, s, idx, values, lam, 0.5)
+        want = _brute_decide(p_m, s, idx, values, lam, 0.5)
+        assert (int(got[0][0]), float(got[1][0]), int(got[2][0]), int(got[3][0])) == want
+
+
+def test_decide_without_matching_neighbour_emits_the_token():
+    values = np.array([1, 1, 2], dtype=np.int32)
+    p_m = np.array([0.7, 0.2, 0.1])
+    tok, pmax, key, use = oracle.decide(p_m, np.array([-1.0, -2.0]), np.array([0, 2]), values,
+                                        0.1, 0.5)
+    assert tok[0] == 0 and pmax[0] == 0.7 and key[0] == -1 and use[0] == 0
+
+
+@pytest.mark.parametrize("lam,delta,want", [(0.2, 0.5, 1), (0.5, 0.5, 1), (0.51, 0.5, 0)])
+def test_decide_span_rule_of_eq6(lam, delta, want):
+    values = np.array([3, 0, 3], dtype=np.int32)
+    p_m = np.array([0.1, 0.1, 0.1, 0.7])
+    _, _, key, use = oracle.decide(p_m, np.array([-4.0, -1.0, -3.0]), np.array([0, 1, 2]),
+                                   values, lam, delta)
+    assert key[0] == 2 and use[0] == want  # nearest neighbour with token 3 is key 2
+
+
+# ---------------------------------------------------------------- Eq. 7
+
+def _frac(e):
+    return float(eval(e, {"__builtins__": {}}, {}))
+
+
+def test_verify_hand_worked_example():
+    with open(os.path.join(GOLDEN, "verify_hand.json")) as f:
+        g = json.load(f)
+    ratio, acc, n_acc = oracle.verify(np.array(g["p_m"]), np.array(g["draft"]),
+                                      np.array(g["span_off"]), g["gamma"])
+    np.testing.assert_allclose(ratio, [_frac(e) for e in g["expect_ratio"]], rtol=1e-15)
+    assert acc.tolist() == g["expect_accept"]
+    assert n_acc.tolist() == g["expect_n_accept"]
+
+
+def test_verify_closed_forms():
+    rng = np.random.default_rng(31)
+    V = 50
+    p = rng.dirichlet(np.ones(V), 6)
+    draft = p.argmax(1).astype(np.int32)  # drafting the argmax: ratio = 1/gamma
+    ratio, acc, n = oracle.verify(p, draft, np.array([0, 6]), 0.05)
+    np.testing.assert_allclose(ratio, 20.0, rtol=1e-14)
+    assert acc.all() and n[0] == 6
+    # a token with zero probability is always rejected and cuts the span there
+    p2 = p.copy()
+    p2[3, draft[3]] = 0.0
+    _, acc2, n2 = oracle.verify(p2, draft, np.array([0, 6]), 0.05)
+    assert acc2[3] == 0 and n2[0] == 3
+    # gamma = 1: accept iff the draft has more than half the top probability
+    q = np.array([[0.4, 0.3, 0.3], [0.4, 0.21, 0.39], [0.4, 0.2, 0.4]])
+    _, acc3, _ = oracle.verify(q, np.array([1, 1, 1]), np.array([0, 3]), 1.0)
+    assert acc3.tolist() == [1, 1, 0]
+
+
+# ---------------------------------------------------------------- masked keys
+
+def test_search_with_excluded_keys_is_search_of_the_rest():
+    rng = np.random.default_rng(32)
+    K = rng.standard_normal((400, 10)).astype(np.float32)
+    q = rng.standard_normal((3, 10)).astype(np.float32)
+    excl = rng.random(400) < 0.3
+    s, I = oracle.knn_search(K, q, 25, exclude=excl)
+    keep = np.flatnonzero(~excl)
+    D = cdist(q.astype(np.float64), K[keep].astype(np.float64), "sqeuclidean")
+    for b in range(3):
+        want = sorted((float(D[b, j]), int(keep[j])) for j in range(len(keep)))[:25]
+        assert I[b].tolist() == [i for _, i in want]
+        np.testing.assert_array_equal(-s[b], [dd for dd, _ in want])
+    # ragged: the exclusion applies inside segments too
+    off = np.array([0, 150, 150, 400])
+    s2, I2 = oracle.knn_search(K, q, 10, seg_off=off, exclude=excl)
+    assert not np.isin(I2[I2 >= 0], np.flatnonzero(excl)).any()
+    assert (I2[1] == -1).all()
