@@ -210,6 +210,78 @@ NEST_API nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_
                             void* stream);
 
 /*
+ * nest_knn_search over the keys not yet used in this generation: accepted
+ * spans are masked out of the datastore and never retrieved again
+ * (Sec. 3.4, last paragraph).
+ *
+ *   key_mask  ceil(N / 32) uint32 words on the device; bit (k % 32) of word
+ *             k / 32 set means key k is never a candidate.  Owned by the
+ *             caller (nest_mask_keys sets bits).
+ * Other arguments and outputs are those of nest_knn_search.
+ */
+NEST_API nest_status_t nest_knn_search_masked(nest_datastore_t* ds, const void* q, int32_t B,
+                                              int32_t r, const int64_t* seg_off,
+                                              const uint32_t* key_mask, float* s_out,
+                                              int64_t* idx_out, void* stream);
+
+/*
+ * Mark keys [first_key, first_key + count) as used in key_mask (atomic OR on
+ * the device, stream-ordered): the keys of an accepted span, which are
+ * consecutive in a passage's datastore.  0 <= first_key <= N - count.
+ */
+NEST_API nest_status_t nest_mask_keys(nest_datastore_t* ds, uint32_t* key_mask, int64_t first_key,
+                                      int64_t count, void* stream);
+
+/*
+ * Greedy token, span start and span decision for each row b < B (Eq. 5 and
+ * Eq. 6, Sec. 3.3; the span-selection steps of Algorithm 1):
+ *
+ *   token_out[b]    = argmax_w p_m[b][w]             (ties: smaller token id)
+ *   p_max_out[b]    = p_m[b][token_out[b]]
+ *   span_key_out[b] = the key index of the neighbour i of row b with
+ *                     V[idx_i] = token whose own term exp(mu s_i) is largest,
+ *                     i.e. the nearest such neighbour (ties: smaller key
+ *                     index): the start of the n-gram continuation in the
+ *                     corpus; -1 if no neighbour has that value.  (Eq. 5 and
+ *                     Algorithm 1 write an argmax of p_kNN over neighbours
+ *                     with value w_t, which is one shared number; the
+ *                     max-pooling is read as pooling their own terms.)
+ *   use_span_out[b] = 1 if lambda[b] <= delta and a span start exists (Eq. 6
+ *                     emits the n-gram), else 0 (emit the token).
+ *
+ *   p_m        B x vocab fp32 (for example from nest_knn_mix_rrc).
+ *   s_in/idx_in  B x r neighbours from the search.
+ *   lambda     B fp32 per-row interpolation weights (lambda_t of Eq. 4).
+ */
+NEST_API nest_status_t nest_knn_decide(nest_datastore_t* ds, const float* p_m, const float* s_in,
+                                       const int64_t* idx_in, const float* lambda, int32_t B,
+                                       int32_t r, float delta, int32_t* token_out,
+                                       float* p_max_out, int64_t* span_key_out,
+                                       int32_t* use_span_out, void* stream);
+
+/*
+ * Relaxed speculative decoding of drafted spans (Eq. 7, Sec. 3.4; the
+ * verification loop of Algorithm 1).  Row b of p_m (rows x vocab fp32) is
+ * p_M at draft position b given the prefix and the drafted tokens before
+ * it; draft[b] is the token drafted there.  Span j covers rows
+ * [span_off[j], span_off[j+1]) (spans + 1 int32 offsets).
+ *
+ *   ratio_out[b]    = p_m[b][draft[b]] / (gamma * max_w p_m[b][w])  (0 if the max is 0)
+ *   accept_out[b]   = 1 if min(1, ratio) > 1/2, else 0 (Algorithm 1 stops at
+ *                     the first position whose acceptance is at most 1/2)
+ *   n_accept_out[j] = number of leading accepted positions of span j
+ *
+ * gamma in (0, 1] is the relaxation factor.  A draft token outside
+ * [0, vocab) is rejected and recorded as NEST_ERR_VALUE_RANGE; bad span
+ * offsets give n_accept = 0 and NEST_ERR_INVALID_ARG in the device status.
+ */
+NEST_API nest_status_t nest_verify_spans(nest_datastore_t* ds, const float* p_m,
+                                         const int32_t* draft, int32_t rows,
+                                         const int32_t* span_off, int32_t spans, float gamma,
+                                         float* ratio_out, int32_t* accept_out,
+                                         int32_t* n_accept_out, void* stream);
+
+/*
  * Synchronize `stream`, return the first condition the GPU recorded for
  * this datastore since the previous call (NEST_OK if none), and clear it.
  */

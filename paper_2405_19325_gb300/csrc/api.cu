@@ -287,8 +287,8 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
 // Large query batches: [sample pass, selection of the sample,] thresholded
 // pass over all keys, exact selection of the survivors.
 nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* q, int32_t B,
-                          int32_t r, float* s_out, int64_t* idx_out, uint64_t* scratch, bool timed,
-                          cudaStream_t stream)
+                          int32_t r, const uint32_t* key_mask, float* s_out, int64_t* idx_out,
+                          uint64_t* scratch, bool timed, cudaStream_t stream)
 {
     nest_status_t st;
     int32_t* cnt = reinterpret_cast<int32_t*>(scratch + sp.off_cnt);
@@ -300,6 +300,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     WideArgs wa{};
     wa.knorm = ds->knorm;
     wa.q = q;
+    wa.key_mask = key_mask;
     wa.status = ds->status;
     wa.r = r;
     wa.d = ds->d;
@@ -385,9 +386,9 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
 // (64-bit words) is the handle's own or the caller's; timing events are
 // recorded around the scan when `timed`.
 nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
-                            const int64_t* seg_off, float* s_out, int64_t* idx_out,
-                            uint64_t* scratch, size_t scratch_words, bool timed,
-                            cudaStream_t stream)
+                            const int64_t* seg_off, const uint32_t* key_mask, float* s_out,
+                            int64_t* idx_out, uint64_t* scratch, size_t scratch_words,
+                            bool timed, cudaStream_t stream)
 {
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
@@ -397,7 +398,8 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
     uint64_t* regionB = scratch + sp.cand_words;
 
     cudaError_t e;
-    if (sp.wide) return launch_wide(ds, sp, q, B, r, s_out, idx_out, scratch, timed, stream);
+    if (sp.wide)
+        return launch_wide(ds, sp, q, B, r, key_mask, s_out, idx_out, scratch, timed, stream);
     if (sp.tc) {
         CUtensorMap qmap;
         if (!encode_bf16_rows(&qmap, q, B, ds->d, 16, false)) return NEST_ERR_CUDA;
@@ -405,6 +407,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         ta.knorm = ds->knorm;
         ta.q = q;
         ta.seg_off = seg_off;
+        ta.key_mask = key_mask;
         ta.cand = regionA;
         ta.status = ds->status;
         ta.N = ds->N;
@@ -424,6 +427,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         sa.knorm = ds->knorm;
         sa.q = q;
         sa.seg_off = seg_off;
+        sa.key_mask = key_mask;
         sa.cand = regionA;
         sa.status = ds->status;
         sa.N = ds->N;
@@ -472,15 +476,15 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
 
 nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
                          const int64_t* seg_off, float* s_out, int64_t* idx_out,
-                         cudaStream_t stream)
+                         cudaStream_t stream, const uint32_t* key_mask = nullptr)
 {
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
     if (st != NEST_OK) return st;
     st = ensure_scratch(ds, sp.cand_words + sp.level_words);
     if (st != NEST_OK) return st;
-    return launch_search(ds, q, B, r, seg_off, s_out, idx_out, ds->scratch, ds->scratch_words,
-                         ds->timing, stream);
+    return launch_search(ds, q, B, r, seg_off, key_mask, s_out, idx_out, ds->scratch,
+                         ds->scratch_words, ds->timing, stream);
 }
 
 nest_status_t run_mix(nest_datastore* ds, const float* s_in, const int64_t* idx_in,
@@ -656,6 +660,94 @@ nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_t B, int3
                    p_m_out, s);
 }
 
+nest_status_t nest_knn_search_masked(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                                     const int64_t* seg_off, const uint32_t* key_mask,
+                                     float* s_out, int64_t* idx_out, void* stream)
+{
+    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st != NEST_OK) return st;
+    if (!key_mask) return NEST_ERR_INVALID_ARG;
+    if (!aligned(key_mask, 4)) return NEST_ERR_ALIGN;
+    return run_search(ds, q, B, r, seg_off, s_out, idx_out, as_stream(stream), key_mask);
+}
+
+nest_status_t nest_mask_keys(nest_datastore_t* ds, uint32_t* key_mask, int64_t first_key,
+                             int64_t count, void* stream)
+{
+    if (!ds || !key_mask || first_key < 0 || count < 0 || first_key > ds->N - count)
+        return NEST_ERR_INVALID_ARG;
+    if (!aligned(key_mask, 4)) return NEST_ERR_ALIGN;
+    const cudaError_t e = launch_mask(key_mask, first_key, count, as_stream(stream));
+    if (e != cudaSuccess) return from_cuda(e);
+    if (count > 0) ++ds->launches;
+    return NEST_OK;
+}
+
+nest_status_t nest_knn_decide(nest_datastore_t* ds, const float* p_m, const float* s_in,
+                              const int64_t* idx_in, const float* lambda, int32_t B, int32_t r,
+                              float delta, int32_t* token_out, float* p_max_out,
+                              int64_t* span_key_out, int32_t* use_span_out, void* stream)
+{
+    if (!ds || !p_m || !s_in || !idx_in || !lambda || !token_out || !p_max_out || !span_key_out ||
+        !use_span_out)
+        return NEST_ERR_INVALID_ARG;
+    if (B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R || delta != delta) return NEST_ERR_INVALID_ARG;
+    if (!aligned(p_m, 4) || !aligned(s_in, 4) || !aligned(idx_in, 8) || !aligned(lambda, 4) ||
+        !aligned(token_out, 4) || !aligned(p_max_out, 4) || !aligned(span_key_out, 8) ||
+        !aligned(use_span_out, 4))
+        return NEST_ERR_ALIGN;
+    DecideArgs a{};
+    a.p_m = p_m;
+    a.s = s_in;
+    a.idx = idx_in;
+    a.V = ds->V;
+    a.lambda = lambda;
+    a.status = ds->status;
+    a.N = ds->N;
+    a.vocab = ds->vocab;
+    a.B = B;
+    a.r = r;
+    a.delta = delta;
+    a.token = token_out;
+    a.p_max = p_max_out;
+    a.span_key = span_key_out;
+    a.use_span = use_span_out;
+    const cudaError_t e = launch_decide(a, as_stream(stream));
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
+    return NEST_OK;
+}
+
+nest_status_t nest_verify_spans(nest_datastore_t* ds, const float* p_m, const int32_t* draft,
+                                int32_t rows, const int32_t* span_off, int32_t spans, float gamma,
+                                float* ratio_out, int32_t* accept_out, int32_t* n_accept_out,
+                                void* stream)
+{
+    if (!ds || !p_m || !draft || !span_off || !ratio_out || !accept_out || !n_accept_out)
+        return NEST_ERR_INVALID_ARG;
+    if (rows < 1 || rows > kMaxB || spans < 1 || spans > rows || !(gamma > 0.f))
+        return NEST_ERR_INVALID_ARG;
+    if (!aligned(p_m, 4) || !aligned(draft, 4) || !aligned(span_off, 4) || !aligned(ratio_out, 4) ||
+        !aligned(accept_out, 4) || !aligned(n_accept_out, 4))
+        return NEST_ERR_ALIGN;
+    VerifyArgs a{};
+    a.p_m = p_m;
+    a.draft = draft;
+    a.span_off = span_off;
+    a.status = ds->status;
+    a.vocab = ds->vocab;
+    a.rows = rows;
+    a.spans = spans;
+    a.gamma = gamma;
+    a.ratio = ratio_out;
+    a.accept = accept_out;
+    a.n_accept = n_accept_out;
+    const cudaError_t e = launch_verify(a, as_stream(stream));
+    if (e != cudaSuccess) return from_cuda(e);
+    ds->launches += 2;
+    return NEST_OK;
+}
+
 nest_status_t nest_device_status(nest_datastore_t* ds, void* stream)
 {
     if (!ds) return NEST_ERR_INVALID_ARG;
@@ -747,8 +839,8 @@ nest_status_t search_with_scratch(nest_datastore* ds, const void* q, int32_t B, 
 {
     nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
     if (st != NEST_OK) return st;
-    return launch_search(ds, q, B, r, seg_off, s_out, idx_out, scratch, scratch_words, false,
-                         stream);
+    return launch_search(ds, q, B, r, seg_off, nullptr, s_out, idx_out, scratch, scratch_words,
+                         false, stream);
 }
 
 }  // namespace nest

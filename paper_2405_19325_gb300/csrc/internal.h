@@ -16,6 +16,12 @@ namespace nest {
 // with ties broken by the smaller key index.  kNoCandidate pads lists.
 constexpr uint64_t kNoCandidate = ~0ull;
 
+// Bit k of a key mask set: key k has been used and is never a candidate.
+__device__ __forceinline__ bool key_masked(const uint32_t* mask, int64_t k)
+{
+    return mask != nullptr && ((__ldg(mask + (k >> 5)) >> (k & 31)) & 1u);
+}
+
 // Device status word: the first recorded nest_status_t value wins.
 __device__ __forceinline__ void record_status(int* status, int code)
 {
@@ -49,6 +55,7 @@ struct ScanArgs {
     const float* knorm;
     const void* q;
     const int64_t* seg_off;  // nullptr: full scan
+    const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     uint64_t* cand;          // [groups * parts][nq][r] candidate lists
     int* status;
     int64_t N;
@@ -86,6 +93,7 @@ struct TcScanArgs {
     const float* knorm;
     const void* q;
     const int64_t* seg_off;  // nullptr: full scan
+    const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     uint64_t* cand;          // [groups * parts][nq][r]
     int* status;
     int64_t N;
@@ -117,6 +125,7 @@ struct WidePlan {
 struct WideArgs {
     const float* knorm;
     const void* q;
+    const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     int* status;
     const float* s_sample;  // B x r sample neighbours (threshold = s[r-1]); null: admit all
     int32_t r;
@@ -190,6 +199,43 @@ struct MixArgs {
 };
 
 cudaError_t launch_mix(const MixArgs& args, cudaStream_t stream);
+
+// ---------------------------------------------------------------- decide.cu
+struct DecideArgs {
+    const float* p_m;    // B x vocab
+    const float* s;      // B x r
+    const int64_t* idx;  // B x r
+    const int32_t* V;
+    const float* lambda;  // B
+    int* status;
+    int64_t N;
+    int32_t vocab;
+    int32_t B;
+    int32_t r;
+    float delta;
+    int32_t* token;
+    float* p_max;
+    int64_t* span_key;
+    int32_t* use_span;
+};
+
+struct VerifyArgs {
+    const float* p_m;      // rows x vocab
+    const int32_t* draft;  // rows
+    const int32_t* span_off;  // spans + 1
+    int* status;
+    int32_t vocab;
+    int32_t rows;
+    int32_t spans;
+    float gamma;
+    float* ratio;
+    int32_t* accept;
+    int32_t* n_accept;
+};
+
+cudaError_t launch_decide(const DecideArgs& args, cudaStream_t stream);
+cudaError_t launch_verify(const VerifyArgs& args, cudaStream_t stream);
+cudaError_t launch_mask(uint32_t* mask, int64_t first, int64_t count, cudaStream_t stream);
 
 // ---------------------------------------------------------------- api.cu, for noalloc.cu
 // Scratch words (64-bit) a search of this shape needs; no allocation, no launch.

@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
             dist = (dist <= 0.f) ? 0.f : dist;  // NaN stays NaN and sorts last
             const int64_t row = lo + (int64_t)i * kScanRows + rr;
             key = ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)row;
-            accept = (rr < rows) && (b < nqv) && (key <= sh.thr[b]);
+            accept = (rr < rows) && (b < nqv) && (key <= sh.thr[b]) && !key_masked(a.key_mask, row);
         }
         __syncwarp();
         mbar_arrive(&sh.pempty[ps]);

@@ -237,7 +237,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             tmem_ld_16(tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * kMmaN), acc);
             tc_fence_before();
             mbar_arrive(&sh.acc_empty[buf]);
-            const bool valid = row < hi;
+            const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
 #pragma unroll
             for (int b = 0; b < NQ; ++b) {
                 float dist = fmaf(-2.f, __uint_as_float(acc[b]), qn[b] + kn);

@@ -228,7 +228,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int64_t row = lo + (int64_t)j * kTileM + row_in_tile;
             const float kn = kn_next;
             kn_next = (row + kTileM < hi) ? __ldg(a.knorm + (row + kTileM) * ks) : 0.f;
-            const bool valid = row < hi;
+            const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
             wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
             tc_fence_after();
             const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);

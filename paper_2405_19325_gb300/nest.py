@@ -35,6 +35,10 @@ SIGNATURES = {
     "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
     "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_static": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
+    "nest_knn_search_masked": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P, _P]),
+    "nest_mask_keys": (ctypes.c_int, [_P, _P, _I64, _I64, _P]),
+    "nest_knn_decide": (ctypes.c_int, [_P, _P, _P, _P, _P, _I32, _I32, _F, _P, _P, _P, _P, _P]),
+    "nest_verify_spans": (ctypes.c_int, [_P, _P, _P, _I32, _P, _I32, _F, _P, _P, _P, _P]),
     "nest_knn_mix": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _P, _P, _P]),
     "nest_knn_mix_rrc": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _F, _P, _P, _P, _P]),
     "nest_knn_step": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _F, _F, _P, _P, _P, _P, _P]),
@@ -161,6 +165,71 @@ class Datastore:
                                          _dev(idx_out, "idx_out", torch.int64), _stream(stream)),
                "nest_knn_search")
         return s_out, idx_out
+
+    def new_key_mask(self) -> torch.Tensor:
+        """All-clear key mask (one bit per key, int32 words) on the current device."""
+        return torch.zeros((self.N + 31) // 32, dtype=torch.int32, device="cuda")
+
+    def mask_keys(self, key_mask: torch.Tensor, first_key: int, count: int, stream=None) -> None:
+        """Mark keys [first_key, first_key + count) as used (Sec. 3.4 masking)."""
+        _check(self._lib.nest_mask_keys(self._h, _dev(key_mask, "key_mask", torch.int32),
+                                        int(first_key), int(count), _stream(stream)),
+               "nest_mask_keys")
+
+    def search_masked(self, q: torch.Tensor, r: int, key_mask: torch.Tensor,
+                      seg_off: torch.Tensor | None = None, stream=None):
+        """search() over the keys whose bit in key_mask is clear."""
+        B = q.shape[0]
+        if q.dtype != self.dtype or q.dim() != 2 or q.shape[1] != self.d:
+            raise ValueError("q must be B x d with the datastore's dtype")
+        if key_mask.numel() < (self.N + 31) // 32:
+            raise ValueError("key_mask needs one bit per key")
+        s_out = torch.empty(B, r, dtype=torch.float32, device=q.device)
+        idx_out = torch.empty(B, r, dtype=torch.int64, device=q.device)
+        sp = _dev(seg_off, "seg_off", torch.int64) if seg_off is not None else None
+        _check(self._lib.nest_knn_search_masked(self._h, _dev(q, "q"), B, r, sp,
+                                                _dev(key_mask, "key_mask", torch.int32),
+                                                s_out.data_ptr(), idx_out.data_ptr(),
+                                                _stream(stream)),
+               "nest_knn_search_masked")
+        return s_out, idx_out
+
+    def decide(self, p_m: torch.Tensor, s: torch.Tensor, idx: torch.Tensor, lam: torch.Tensor,
+               delta: float, stream=None) -> dict:
+        """Eq. 5 / Eq. 6: greedy token, its probability, span start key, span choice."""
+        B, r = s.shape
+        self._check_rows(p_m, B)
+        dev = p_m.device
+        o = {"token": torch.empty(B, dtype=torch.int32, device=dev),
+             "p_max": torch.empty(B, dtype=torch.float32, device=dev),
+             "span_key": torch.empty(B, dtype=torch.int64, device=dev),
+             "use_span": torch.empty(B, dtype=torch.int32, device=dev)}
+        _check(self._lib.nest_knn_decide(self._h, _dev(p_m, "p_m", torch.float32),
+                                         _dev(s, "s", torch.float32), _dev(idx, "idx", torch.int64),
+                                         _dev(lam, "lambda", torch.float32), B, r, float(delta),
+                                         o["token"].data_ptr(), o["p_max"].data_ptr(),
+                                         o["span_key"].data_ptr(), o["use_span"].data_ptr(),
+                                         _stream(stream)),
+               "nest_knn_decide")
+        return o
+
+    def verify(self, p_m: torch.Tensor, draft: torch.Tensor, span_off: torch.Tensor, gamma: float,
+               stream=None) -> dict:
+        """Eq. 7 over drafted spans: per-row ratio and acceptance, accepted prefix per span."""
+        rows = p_m.shape[0]
+        spans = span_off.numel() - 1
+        dev = p_m.device
+        o = {"ratio": torch.empty(rows, dtype=torch.float32, device=dev),
+             "accept": torch.empty(rows, dtype=torch.int32, device=dev),
+             "n_accept": torch.empty(spans, dtype=torch.int32, device=dev)}
+        _check(self._lib.nest_verify_spans(self._h, _dev(p_m, "p_m", torch.float32),
+                                           _dev(draft, "draft", torch.int32), rows,
+                                           _dev(span_off, "span_off", torch.int32), spans,
+                                           float(gamma), o["ratio"].data_ptr(),
+                                           o["accept"].data_ptr(), o["n_accept"].data_ptr(),
+                                           _stream(stream)),
+               "nest_verify_spans")
+        return o
 
     def mix(self, s: torch.Tensor, idx: torch.Tensor, p_lm: torch.Tensor, mu: float, lam: float,
             want_p_knn: bool = False, p_m_out=None, p_knn_out=None, stream=None):
