@@ -30,6 +30,7 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
 import synth  # noqa: E402
@@ -51,6 +52,10 @@ def parse():
                    help="queries in the oracle's bounded sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=200)
+    p.add_argument("--pipeline", choices=["knnlm", "nest", "verify"], default="knnlm",
+                   help="knnlm: search + Eq. 2 + Eq. 3 (default); nest: masked search + Eq. 2 + "
+                        "Eq. 4 + Eq. 5/6 decision; verify: a batch of drafted positions "
+                        "searched, mixed (Eq. 4) and verified (Eq. 7)")
     p.add_argument("--sweep", default=None,
                    help="comma-separated query batch sizes measured on one datastore, one JSON "
                         "line each (e.g. 1,8,64,256 for the d=8192 workload)")
@@ -287,9 +292,9 @@ def dram_traffic(w, args, kernel):
     return None
 
 
-def config_of(w, x):
+def config_of(w, x, pipeline="knnlm"):
     B = x.q.shape[0]
-    return {"workload": w.name, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
+    return {"workload": w.name, "pipeline": pipeline, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
             "vocab": w.vocab, "key_dtype": w.dtype, "accumulate": "f32",
             "mu": w.mu, "lambda": w.lam,
             "ragged": bool(w.ragged),
@@ -325,15 +330,53 @@ def main():
         dist.destroy_process_group()
 
 
+NEST_ALPHA, NEST_TAU, NEST_DELTA, NEST_GAMMA = 0.3, 0.1, 0.5, 5e-2  # App. A (Wikipedia, 70B)
+
+
+def make_step(args, w, x, ds):
+    """(step, metric) for the pipeline: step() runs one pass of the hot path."""
+    if args.pipeline == "knnlm":
+        out = {}
+
+        def step():
+            ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off, out=out)
+            return out["p_m"]
+        return step, "queries/s for fused kNN search+top-r+p_M mix"
+    B = x.q.shape[0]
+    mask = ds.new_key_mask()
+    # keys of previously accepted spans: every 64th run of 64 keys is used
+    words = mask.cpu().numpy().view(np.uint32)
+    words[::64] = np.uint32(0xFFFFFFFF)
+    words[1::64] = np.uint32(0xFFFFFFFF)
+    mask.copy_(torch.from_numpy(words.view(np.int32)))
+    if args.pipeline == "nest":
+        def step():
+            s, idx = ds.search_masked(x.q, w.r, mask, seg_off=x.seg_off)
+            p_m, lam = ds.mix_rrc(s, idx, x.p_lm, w.mu, NEST_ALPHA, NEST_TAU)
+            return ds.decide(p_m, s, idx, lam, NEST_DELTA)["token"]
+        return step, ("queries/s for NEST step (masked kNN search+top-r+p_M with RRC lambda_t+"
+                      "greedy token/span decision)")
+    draft = torch.randint(0, w.vocab, (B,), dtype=torch.int32, device=x.q.device)
+    span_off = torch.tensor([0, B], dtype=torch.int32, device=x.q.device)
+
+    def step():
+        s, idx = ds.search_masked(x.q, w.r, mask, seg_off=x.seg_off)
+        p_m, lam = ds.mix_rrc(s, idx, x.p_lm, w.mu, NEST_ALPHA, NEST_TAU)
+        return ds.verify(p_m, draft, span_off, NEST_GAMMA)["n_accept"]
+    return step, ("draft positions/s for NEST span verification (kNN search+top-r+p_M with RRC "
+                  "lambda_t+relaxed speculative acceptance) of one drafted span")
+
+
 def measure(args, w, x_all, ds, B, world, rank, local):
     """Time one batch size on an existing datastore; returns the JSON line (rank 0)."""
     x = synth.Inputs(K=x_all.K, V=x_all.V, q=x_all.q[:B].contiguous(),
                      p_lm=x_all.p_lm[:B].contiguous(),
                      seg_off=x_all.seg_off[:B + 1].contiguous() if x_all.seg_off is not None else None)
-    out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off)  # allocates scratch once
+    step, metric = make_step(args, w, x, ds)
+    step()  # allocates scratch once
     stream = torch.cuda.current_stream()
     for _ in range(max(3, args.warmup)):
-        ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off, out=out)
+        step()
     torch.cuda.synchronize()
     if ds.device_status() != 0:
         raise SystemExit("device status error during warm-up")
@@ -350,7 +393,7 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     for _ in range(args.steps):
-        ds.step(x.q, w.r, x.p_lm, w.mu, w.lam, seg_off=x.seg_off, out=out)
+        step()
     t1.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -400,18 +443,36 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     q_h = x.q.cpu().pin_memory()
     p_h = x.p_lm.cpu().pin_memory()
     so_h = x.seg_off.cpu().pin_memory() if x.seg_off is not None else None
-    staging = {}
+    h2d = q_h.numel() * q_h.element_size() + p_h.numel() * 4 + (
+        so_h.numel() * 8 if so_h is not None else 0)
+    if args.pipeline == "knnlm":
+        staging = {}
+
+        def e2e_step():
+            ds.step_host(q_h, w.r, p_h, w.mu, w.lam, seg_off_host=so_h, staging=staging)
+        d2h = B * w.vocab * 4 + B * w.r * 4 + B * w.r * 8
+    else:
+        # inputs copied into the tensors the step reads, the step's decision read back
+        res = step()
+        res_h = torch.empty(res.shape, dtype=res.dtype).pin_memory()
+
+        def e2e_step():
+            x.q.copy_(q_h, non_blocking=True)
+            x.p_lm.copy_(p_h, non_blocking=True)
+            if so_h is not None:
+                x.seg_off.copy_(so_h, non_blocking=True)
+            res_h.copy_(step(), non_blocking=True)
+            stream.synchronize()
+        d2h = res_h.numel() * res_h.element_size()
     for _ in range(3):
-        ds.step_host(q_h, w.r, p_h, w.mu, w.lam, seg_off_host=so_h, staging=staging)
+        e2e_step()
     barrier(world)
     te = time.perf_counter()
     for _ in range(args.e2e_steps):
-        ds.step_host(q_h, w.r, p_h, w.mu, w.lam, seg_off_host=so_h, staging=staging)
+        e2e_step()
     e2e_s = max_over_ranks(time.perf_counter() - te, world)
-    h2d = q_h.numel() * q_h.element_size() + p_h.numel() * 4 + (
-        so_h.numel() * 8 if so_h is not None else 0)
-    d2h = B * w.vocab * 4 + B * w.r * 4 + B * w.r * 8
-    e2e = {"value": world * B * args.e2e_steps / e2e_s, "unit": "queries/s",
+    e2e = {"value": world * B * args.e2e_steps / e2e_s,
+           "unit": "positions/s" if args.pipeline == "verify" else "queries/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     cpu = None
@@ -422,11 +483,11 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     line = None
     if rank == 0:
         line = {
-            "metric": "queries/s for fused kNN search+top-r+p_M mix", "value": value,
-            "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "metric": metric, "value": value,
+            "unit": "positions/s" if args.pipeline == "verify" else "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
-            "data": "synthetic", "config": config_of(w, x),
+            "data": "synthetic", "config": config_of(w, x, args.pipeline),
             "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clk,

@@ -57,6 +57,11 @@ WORKLOADS = {
     # large query batch over 4M keys
     "large_batch": Workload("large_batch", "bf16", 4096, 1 << 22, 512, 256, 32000, 1 / 64, 0.8,
                             3.0, centres=256),
+    # NEST verification of one drafted span: the on-the-fly datastore K' of one
+    # query (40 passages x 256 tokens around 40 passage centres) searched by the
+    # n = 64 drafted positions at once (App. A: n-gram length 64, top-1024)
+    "nest_span": Workload("nest_span", "bf16", 4096, 40 * 256, 64, 1024, 32000, 1 / 64, 0.8, 3.0,
+                          centres=40),
     # 70B hidden size over 8M keys (128 GiB); B is swept over 1, 8, 64, 256
     "hidden8192": Workload("hidden8192", "bf16", 8192, 1 << 23, 1, 1024, 32000,
                            1 / math.sqrt(8192), 0.8, 3.0, centres=256),
