@@ -148,6 +148,11 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+def aggregate(world: int, per_rank_units: int, steps: int, max_ms: float) -> float:
+    """Whole-job throughput: units processed by all ranks over the slowest rank's time."""
+    return world * per_rank_units * steps / (max_ms / 1e3)
+
+
 def host_keys(K: torch.Tensor, rows: int | None = None):
     """Exact bytes of the first ``rows`` keys on the host (bf16 as uint16), ~1 GiB pieces."""
     import numpy as np
@@ -405,7 +410,7 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     if ds.device_status() != 0:
         raise SystemExit("device status error during the timed steps")
     ms = max_over_ranks(ms_local, world)
-    value = world * B * args.steps / (ms / 1e3)
+    value = aggregate(world, B, args.steps, ms)
 
     # ---- roofline of the dominant kernel (the key scan)
     esize = 2 if w.dtype == "bf16" else 4
