@@ -62,6 +62,8 @@ struct SearchPlan {
     int nq, groups, parts;
     size_t cand_words;   // scan output: groups * parts * nq * r
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
+    size_t cnt_words;    // list lengths of the scan output and of the merge levels
+    size_t total_words;  // all scratch of the search
     // Large query batches (tc_wide.cu): sample pass + thresholded pass.
     bool wide;
     WidePlan wps, wpm;        // sample pass, main pass
@@ -149,6 +151,9 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
     const int per = merge_lists_per_cta(r);
     const int lvl1 = (sp->parts + per - 1) / per;
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
+    // int32 counts: [groups * parts * nq] then [B * lvl1], as 64-bit words
+    sp->cnt_words = ((size_t)sp->groups * sp->parts * sp->nq + 1) / 2 + ((size_t)B * lvl1 + 1) / 2;
+    sp->total_words = sp->cand_words + sp->level_words + sp->cnt_words;
     sp->wide = false;
     // More queries than one CTA can keep lists for: stream the keys once per
     // group of up to 256 queries against sampled admission thresholds.
@@ -177,6 +182,8 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             sp->wide = true;
             sp->cand_words = sp->wide_words;
             sp->level_words = 0;
+            sp->cnt_words = 0;
+            sp->total_words = sp->wide_words;
         }
     }
     return NEST_OK;
@@ -393,9 +400,11 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
     if (st != NEST_OK) return st;
-    if (sp.cand_words + sp.level_words > scratch_words) return NEST_ERR_OVERFLOW;
+    if (sp.total_words > scratch_words) return NEST_ERR_OVERFLOW;
     uint64_t* regionA = scratch;
     uint64_t* regionB = scratch + sp.cand_words;
+    int32_t* cntA = reinterpret_cast<int32_t*>(scratch + sp.cand_words + sp.level_words);
+    int32_t* cntB = cntA + ((size_t)sp.groups * sp.parts * sp.nq + 1) / 2 * 2;
 
     cudaError_t e;
     if (sp.wide)
@@ -409,6 +418,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         ta.seg_off = seg_off;
         ta.key_mask = key_mask;
         ta.cand = regionA;
+        ta.cand_cnt = cntA;
         ta.status = ds->status;
         ta.N = ds->N;
         ta.d = ds->d;
@@ -429,6 +439,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         sa.seg_off = seg_off;
         sa.key_mask = key_mask;
         sa.cand = regionA;
+        sa.cand_cnt = cntA;
         sa.status = ds->status;
         sa.N = ds->N;
         sa.row_bytes = ds->row_bytes;
@@ -448,6 +459,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
 
     MergeArgs ma{};
     ma.in = regionA;
+    ma.in_cnt = cntA;
     ma.list_stride = (int64_t)sp.nq * r;
     ma.nq_in = sp.nq;
     ma.lists = sp.parts;
@@ -461,11 +473,13 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
         const bool last = groups == 1;
         ma.out = into_b ? regionB : regionA;
+        ma.out_cnt = into_b ? cntB : cntA;
         e = launch_merge(ma, last, stream);
         if (e != cudaSuccess) return from_cuda(e);
         ++ds->launches;
         if (last) break;
         ma.in = ma.out;
+        ma.in_cnt = ma.out_cnt;
         ma.list_stride = r;
         ma.nq_in = 1;
         ma.lists = groups;
@@ -481,7 +495,7 @@ nest_status_t run_search(nest_datastore* ds, const void* q, int32_t B, int32_t r
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
     if (st != NEST_OK) return st;
-    st = ensure_scratch(ds, sp.cand_words + sp.level_words);
+    st = ensure_scratch(ds, sp.total_words);
     if (st != NEST_OK) return st;
     return launch_search(ds, q, B, r, seg_off, key_mask, s_out, idx_out, ds->scratch,
                          ds->scratch_words, ds->timing, stream);
@@ -513,7 +527,8 @@ nest_status_t run_mix(nest_datastore* ds, const float* s_in, const int64_t* idx_
     // Enough CTAs to stream the vocabulary rows, at least one per query.
     const int64_t want = std::max<int64_t>(1, (2LL * ds->num_sms + B - 1) / B);
     const int64_t by_vocab = std::max<int64_t>(1, ds->vocab / 2048);
-    m.slices = (int32_t)std::min<int64_t>(want, by_vocab);
+    m.slices = (int32_t)std::max<int64_t>(mix_min_slices(ds->vocab),
+                                          std::min<int64_t>(want, by_vocab));
     cudaError_t e = launch_mix(m, stream);
     if (e != cudaSuccess) return from_cuda(e);
     ++ds->launches;
@@ -605,7 +620,7 @@ nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_B, int32_
         for (int B = 1; B <= max_B; B = (B == max_B) ? max_B + 1 : std::min(max_B, B * 2)) {
             SearchPlan sp;
             if (plan_search(ds, B, r, ragged != 0, &sp) == NEST_OK)
-                need = std::max(need, sp.cand_words + sp.level_words);
+                need = std::max(need, sp.total_words);
         }
     }
     return ensure_scratch(ds, need);
@@ -829,7 +844,7 @@ nest_status_t search_scratch_words(const nest_datastore* ds, int32_t B, int32_t 
     SearchPlan sp;
     nest_status_t st = plan_search(ds, B, r, ragged, &sp);
     if (st != NEST_OK) return st;
-    *words = sp.cand_words + sp.level_words;
+    *words = sp.total_words;
     return NEST_OK;
 }
 

@@ -57,6 +57,7 @@ struct ScanArgs {
     const int64_t* seg_off;  // nullptr: full scan
     const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     uint64_t* cand;          // [groups * parts][nq][r] candidate lists
+    int32_t* cand_cnt;       // [groups * parts][nq] real entries of each list
     int* status;
     int64_t N;
     int32_t row_bytes;
@@ -95,6 +96,7 @@ struct TcScanArgs {
     const int64_t* seg_off;  // nullptr: full scan
     const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     uint64_t* cand;          // [groups * parts][nq][r]
+    int32_t* cand_cnt;       // [groups * parts][nq] real entries of each list
     int* status;
     int64_t N;
     int32_t d;
@@ -160,14 +162,17 @@ cudaError_t launch_gselect(const GselectArgs& args, cudaStream_t stream);
 // ---------------------------------------------------------------- merge.cu
 // Merge candidate lists of each query into its top r.
 struct MergeArgs {
-    const uint64_t* in;    // candidate lists
-    int64_t list_stride;   // entries between consecutive lists of one query
-    int32_t nq_in;         // query b's first list is at ((b / nq_in) * lists * nq_in + b % nq_in) * r
+    const uint64_t* in;    // candidate lists; list (b, l) starts at (base(b) + l * nq_in) * r with
+                           // base(b) = (b / nq_in) * lists * nq_in + b % nq_in
+    const int32_t* in_cnt; // real entries of list (b, l), at base(b) + l * nq_in
+    int64_t list_stride;   // entries between consecutive lists of one query (nq_in * r)
+    int32_t nq_in;
     int32_t lists;         // lists per query
     int32_t per_cta;       // lists merged by one CTA
     int32_t B;
     int32_t r;
     uint64_t* out;         // next level: [B][ceil(lists / per_cta)][r]; unused on the last level
+    int32_t* out_cnt;      // next level: [B][ceil(lists / per_cta)]
     float* s_out;          // last level only: B x r
     int64_t* idx_out;      // last level only: B x r
 };
@@ -199,6 +204,7 @@ struct MixArgs {
 };
 
 cudaError_t launch_mix(const MixArgs& args, cudaStream_t stream);
+int mix_min_slices(int vocab);  // slices needed so each fits the shared-memory sums
 
 // ---------------------------------------------------------------- decide.cu
 struct DecideArgs {

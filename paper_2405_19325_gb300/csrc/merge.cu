@@ -1,8 +1,9 @@
 // merge.cu -- combine per-CTA candidate lists into each query's r nearest
 // neighbours (the selection of pi, Sec. 2.2 / Algorithm 1's search step).
 //
-// A CTA loads up to per_cta lists of one query into shared memory (dropping
-// empty slots), keeps the r smallest words with the same radix select the
+// A CTA copies the real entries of up to per_cta lists of one query into
+// shared memory (list lengths come with the lists, so the copy is one fully
+// parallel pass), keeps the r smallest words with the same radix select the
 // scan uses, and either writes them as one list for the next level or, on
 // the last level, sorts them (bitonic) and writes s = -distance and the key
 // index, nearest first, ties by smaller index, padding with (-inf, -1).
@@ -17,11 +18,13 @@ namespace {
 
 constexpr int kMergeThreads = 1024;
 constexpr size_t kMergeBufBytes = 192 * 1024;
+constexpr int kMaxListsPerCta = 1024;
 
 struct MergeShared {
     uint64_t thr;
     int cnt;
-    int wcnt[2][kMergeThreads / 32];
+    int off[kMaxListsPerCta + 1];  // exclusive prefix of the list lengths
+    int wsum[kMergeThreads / 32];
     SelectSmem<kMergeThreads, 1> sel;
 };
 
@@ -47,46 +50,67 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int b = blockIdx.y, grp = blockIdx.x;
     const int l0 = grp * a.per_cta;
-    const int l1 = min(a.lists, l0 + a.per_cta);
-    const uint64_t* src =
-        a.in + ((int64_t)(b / a.nq_in) * a.lists * a.nq_in + b % a.nq_in) * (int64_t)a.r;
+    const int nl = min(a.lists, l0 + a.per_cta) - l0;
+    const int64_t base = (int64_t)(b / a.nq_in) * a.lists * a.nq_in + b % a.nq_in;
+    const uint64_t* src = a.in + base * (int64_t)a.r;
 
-    // Load the lists, keeping real candidates only, in list order.
-    const int total = (l1 - l0) * a.r;
-    int n = 0;
-    for (int base = 0, t = 0; base < total; base += kMergeThreads, ++t) {
-        const int j = base + tid;
-        uint64_t e = kNoCandidate;
-        if (j < total) {
-            const int l = l0 + j / a.r, k = j - (j / a.r) * a.r;
-            e = src[(int64_t)l * a.list_stride + k];
-        }
-        const bool keep = e != kNoCandidate;
-        const uint32_t bal = __ballot_sync(~0u, keep);
-        if (lane == 0) sh.wcnt[t & 1][warp] = __popc(bal);
-        __syncthreads();
-        int before = 0, tot = 0;
+    // exclusive prefix of this CTA's list lengths (nl <= 1024: one value per thread)
+    int len = 0;
+    if (tid < nl) {
+        len = a.in_cnt[base + (int64_t)(l0 + tid) * a.nq_in];
+        len = len < 0 ? 0 : (len > a.r ? a.r : len);
+    }
+    int incl = len;
 #pragma unroll
-        for (int w = 0; w < kMergeThreads / 32; ++w) {
-            const int c = sh.wcnt[t & 1][w];
-            before += (w < warp) ? c : 0;
-            tot += c;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(~0u, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) sh.wsum[warp] = incl;
+    __syncthreads();
+    int carry = 0;
+    for (int w = 0; w < warp; ++w) carry += sh.wsum[w];
+    if (tid < nl) sh.off[tid] = carry + incl - len;
+    if (tid == kMergeThreads - 1) sh.off[nl] = carry + incl;  // nl <= 1024: total
+    __syncthreads();
+    const int total = sh.off[nl];
+
+    // copy the real entries: entry e of the concatenation belongs to the list
+    // whose offset range holds it (binary search over the offsets)
+    for (int e0 = tid; e0 < total; e0 += 4 * kMergeThreads) {
+        uint64_t v[4];
+        int at[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int e = e0 + u * kMergeThreads;
+            at[u] = e;
+            if (e < total) {
+                int lo = 0, hi = nl;  // find the last l with off[l] <= e
+                while (hi - lo > 1) {
+                    const int mid = (lo + hi) >> 1;
+                    if (sh.off[mid] <= e) lo = mid;
+                    else hi = mid;
+                }
+                v[u] = src[(int64_t)(l0 + lo) * a.list_stride + (e - sh.off[lo])];
+            }
         }
-        if (keep) buf[n + before + __popc(bal & lanemask_lt())] = e;
-        n += tot;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (at[u] < total) buf[at[u]] = v[u];
     }
     if (tid == 0) {
-        sh.cnt = n;
+        sh.cnt = total;
         sh.thr = kNoCandidate;
     }
     __syncthreads();
     select_smallest<kMergeThreads, 1>(buf, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
                                       [] { __syncthreads(); });
-    n = sh.cnt;
+    const int n = sh.cnt;
 
     if constexpr (!LAST) {
         uint64_t* dst = a.out + ((int64_t)b * gridDim.x + grp) * a.r;
         for (int j = tid; j < a.r; j += kMergeThreads) dst[j] = j < n ? buf[j] : kNoCandidate;
+        if (tid == 0) a.out_cnt[(int64_t)b * gridDim.x + grp] = n;
     } else {
         const int P2 = next_pow2(n > 0 ? n : 1);
         for (int j = n + tid; j < P2; j += kMergeThreads) buf[j] = kNoCandidate;
@@ -126,7 +150,8 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
 
 int merge_lists_per_cta(int r)
 {
-    const int per = (int)(kMergeBufBytes / ((size_t)r * 8));
+    int per = (int)(kMergeBufBytes / ((size_t)r * 8));
+    per = per > kMaxListsPerCta ? kMaxListsPerCta : per;
     return per < 2 ? 2 : per;
 }
 

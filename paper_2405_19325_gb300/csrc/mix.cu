@@ -2,14 +2,13 @@
 // lambda mix) or Eq. 4 (relative retrieval confidence lambda_t) for each
 // query row.
 //
-// Grid (slices, B).  Every CTA of a row gathers the row's r neighbours'
-// token ids V[idx], forms the softmax weights exp(mu (s_i - s_max)) and
-// their sum Z (a fixed-order reduction), and sorts (token, slot) pairs so
-// that equal tokens are adjacent; it then writes its vocabulary slice:
-// p_M[w] = lambda p_LM[w] everywhere, and, after a block barrier, the
-// entries of the slice that received neighbour mass,
-// p_M[v] = lambda p_LM[v] + (1 - lambda) p_kNN[v].  Sums over equal tokens
-// run in slot order, so results do not depend on scheduling.
+// Grid (slices, B).  Every CTA of a row reads the row's r neighbours,
+// gathers their token ids V[idx], and forms the softmax weights
+// w_i = exp(mu (s_i - s_max)) / Z.  Weights of tokens inside the CTA's
+// vocabulary slice are summed per token in shared memory as 48-bit fixed
+// point: integer addition is associative, so the sums do not depend on the
+// order of the atomics and are exact to 2^-49 per term.  One streaming pass
+// over the slice then writes p_M[w] = lambda p_LM[w] + (1 - lambda) p_kNN[w].
 #include <cmath>
 
 #include "internal.h"
@@ -19,14 +18,10 @@ namespace nest {
 namespace {
 
 constexpr int kMixThreads = 512;
+constexpr int kMixMaxSliceTokens = 16384;  // 128 KiB of fixed-point sums
 constexpr int kWarps = kMixThreads / 32;
-
-__host__ __device__ inline int next_pow2_mix(int x)
-{
-    int p = 1;
-    while (p < x) p <<= 1;
-    return p;
-}
+constexpr float kFixScale = 281474976710656.0f;  // 2^48
+constexpr float kFixInv = 1.0f / 281474976710656.0f;
 
 struct Red {
     float v[kWarps];
@@ -56,10 +51,7 @@ __device__ __forceinline__ float warp_min(float x)
 
 __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
 {
-    extern __shared__ __align__(16) unsigned char smem[];
-    const int P2 = next_pow2_mix(a.r);
-    uint64_t* keys = reinterpret_cast<uint64_t*>(smem);        // P2: (token << 32) | slot
-    float* wts = reinterpret_cast<float*>(keys + P2);          // r: s, then weights
+    extern __shared__ __align__(16) unsigned long long acc[];  // slice tokens, fixed point
     __shared__ Red red;
     __shared__ float bc[4];
     __shared__ int bci;
@@ -74,33 +66,28 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
     const float* s = a.s + (int64_t)b * a.r;
     const int64_t* id = a.idx + (int64_t)b * a.r;
 
-    // Gather token ids, mark real neighbours, and reduce max s, min s, min/max |s|.
+    for (int w = tid; w < w1 - w0; w += kMixThreads) acc[w] = 0ull;
+
+    // Real neighbours: max s, min/max |s|, count (Eq. 2 and Eq. 4 inputs).
     float smax = -INFINITY, amin = INFINITY, amax = 0.f;
     int count = 0;
-    for (int i = tid; i < P2; i += kMixThreads) {
-        uint64_t key = kNoCandidate;
-        if (i < a.r) {
-            const int64_t k = id[i];
-            const float si = s[i];
-            if (k >= 0 && si > -INFINITY) {
-                if (k >= a.N) {
-                    record_status(a.status, NEST_ERR_VALUE_RANGE);
-                } else {
-                    const int32_t v = a.V[k];
-                    if (v < 0 || v >= a.vocab) {
-                        record_status(a.status, NEST_ERR_VALUE_RANGE);
-                    } else {
-                        key = ((uint64_t)(uint32_t)v << 32) | (uint32_t)i;
-                        smax = fmaxf(smax, si);
-                        amin = fminf(amin, fabsf(si));
-                        amax = fmaxf(amax, fabsf(si));
-                        ++count;
-                    }
-                }
-            }
-            wts[i] = si;
+    for (int i = tid; i < a.r; i += kMixThreads) {
+        const int64_t k = id[i];
+        const float si = s[i];
+        if (k < 0 || !(si > -INFINITY)) continue;
+        if (k >= a.N) {
+            record_status(a.status, NEST_ERR_VALUE_RANGE);
+            continue;
         }
-        keys[i] = key;
+        const int32_t v = a.V[k];
+        if (v < 0 || v >= a.vocab) {
+            record_status(a.status, NEST_ERR_VALUE_RANGE);
+            continue;
+        }
+        smax = fmaxf(smax, si);
+        amin = fminf(amin, fabsf(si));
+        amax = fmaxf(amax, fabsf(si));
+        ++count;
     }
     smax = warp_max(smax);
     amin = warp_min(amin);
@@ -132,20 +119,23 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
     smax = bc[0];
     const int nreal = bci;
 
-    // Weights exp(mu (s_i - s_max)) of real neighbours and their sum Z.
+    // Z = sum of exp(mu (s_i - s_max)) over real neighbours (fixed-order tree).
     float zpart = 0.f;
     for (int i = tid; i < a.r; i += kMixThreads) {
-        const float w = keys[i] != kNoCandidate ? expf(a.mu * (wts[i] - smax)) : 0.f;
-        wts[i] = w;
-        zpart += w;
+        const int64_t k = id[i];
+        const float si = s[i];
+        if (k < 0 || k >= a.N || !(si > -INFINITY)) continue;
+        const int32_t v = a.V[k];
+        if (v < 0 || v >= a.vocab) continue;
+        zpart += expf(a.mu * (si - smax));
     }
     zpart = warp_sum(zpart);
     if (lane == 0) red.v[warp] = zpart;
     __syncthreads();
-    float lam = a.lambda;
     if (tid == 0) {
         float z = 0.f;
         for (int w = 0; w < kWarps; ++w) z += red.v[w];
+        float lam = a.lambda;
         if (a.rrc) {
             const float ratio = (bc[2] > 0.f) ? bc[1] / bc[2] : 1.f;
             lam = 1.f / (1.f + expf(-(ratio - a.alpha) / a.tau));
@@ -155,31 +145,27 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
         bc[0] = lam;
         if (a.lam_out != nullptr && slice == 0) a.lam_out[b] = lam;
     }
-
-    // Sort (token, slot) ascending so equal tokens are adjacent, slots in order.
     __syncthreads();
-    for (int k = 2; k <= P2; k <<= 1) {
-        for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int i = tid; i < P2; i += kMixThreads) {
-                const int l = i ^ j;
-                if (l > i) {
-                    const uint64_t x = keys[i], y = keys[l];
-                    if ((x > y) == ((i & k) == 0)) {
-                        keys[i] = y;
-                        keys[l] = x;
-                    }
-                }
-            }
-            __syncthreads();
-        }
-    }
-    lam = bc[0];
+    const float lam = bc[0];
     const float z = bc[3];
 
-    // Dense part of this vocabulary slice.
+    // p_kNN of the slice's tokens: w_i / Z summed per token in fixed point.
+    for (int i = tid; i < a.r; i += kMixThreads) {
+        const int64_t k = id[i];
+        const float si = s[i];
+        if (k < 0 || k >= a.N || !(si > -INFINITY)) continue;
+        const int32_t v = a.V[k];
+        if (v < w0 || v >= w1) continue;
+        const float p = expf(a.mu * (si - smax)) / z;
+        atomicAdd(&acc[v - w0], (unsigned long long)__float2ull_rn(p * kFixScale));
+    }
+    __syncthreads();
+
+    // One pass over the slice: p_M = lambda p_LM + (1 - lambda) p_kNN.
     const float* plm = a.p_lm + (int64_t)b * a.vocab;
     float* pm = a.p_m + (int64_t)b * a.vocab;
     float* pk = a.p_knn ? a.p_knn + (int64_t)b * a.vocab : nullptr;
+    const float one_m = 1.f - lam;
     const bool vec = ((a.vocab & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.p_lm) & 15) == 0) &&
                      ((reinterpret_cast<uintptr_t>(a.p_m) & 15) == 0) &&
                      (pk == nullptr || (reinterpret_cast<uintptr_t>(a.p_knn) & 15) == 0) &&
@@ -188,40 +174,23 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
         const int n4 = (w1 - w0) >> 2;
         const float4* src = reinterpret_cast<const float4*>(plm + w0);
         float4* dst = reinterpret_cast<float4*>(pm + w0);
+        float4* dk = pk ? reinterpret_cast<float4*>(pk + w0) : nullptr;
         for (int i = tid; i < n4; i += kMixThreads) {
-            float4 x = __ldg(src + i);
-            x.x *= lam;
-            x.y *= lam;
-            x.z *= lam;
-            x.w *= lam;
-            dst[i] = x;
-            if (pk) reinterpret_cast<float4*>(pk + w0)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        for (int w = w0 + 4 * n4 + tid; w < w1; w += kMixThreads) {
-            pm[w] = lam * plm[w];
-            if (pk) pk[w] = 0.f;
+            const float4 x = __ldg(src + i);
+            const float k0 = __ull2float_rn(acc[4 * i]) * kFixInv;
+            const float k1 = __ull2float_rn(acc[4 * i + 1]) * kFixInv;
+            const float k2 = __ull2float_rn(acc[4 * i + 2]) * kFixInv;
+            const float k3 = __ull2float_rn(acc[4 * i + 3]) * kFixInv;
+            dst[i] = make_float4(lam * x.x + one_m * k0, lam * x.y + one_m * k1,
+                                 lam * x.z + one_m * k2, lam * x.w + one_m * k3);
+            if (dk) dk[i] = make_float4(k0, k1, k2, k3);
         }
     } else {
         for (int w = w0 + tid; w < w1; w += kMixThreads) {
-            pm[w] = lam * plm[w];
-            if (pk) pk[w] = 0.f;
+            const float kk = __ull2float_rn(acc[w - w0]) * kFixInv;
+            pm[w] = lam * plm[w] + one_m * kk;
+            if (pk) pk[w] = kk;
         }
-    }
-    __syncthreads();
-
-    // Tokens of this slice that received neighbour mass.
-    for (int i = tid; i < P2; i += kMixThreads) {
-        const uint64_t key = keys[i];
-        if (key == kNoCandidate) continue;
-        const uint32_t v = (uint32_t)(key >> 32);
-        if (i > 0 && (uint32_t)(keys[i - 1] >> 32) == v) continue;  // not the first of its token
-        if ((int)v < w0 || (int)v >= w1) continue;
-        float sum = 0.f;
-        for (int j = i; j < P2 && keys[j] != kNoCandidate && (uint32_t)(keys[j] >> 32) == v; ++j)
-            sum += wts[(uint32_t)keys[j]];
-        const float p = sum / z;
-        pm[v] = lam * plm[v] + (1.f - lam) * p;
-        if (pk) pk[v] = p;
     }
 }
 
@@ -229,8 +198,11 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
 
 cudaError_t launch_mix(const MixArgs& a, cudaStream_t stream)
 {
-    const int P2 = next_pow2_mix(a.r);
-    const size_t smem = (size_t)P2 * 8 + (size_t)a.r * 4;
+    // the widest slice of the grid, in tokens
+    const int unit = (a.vocab & 3) == 0 ? 4 : 1;
+    const int64_t units = a.vocab / unit;
+    const int widest = unit * (int)((units + a.slices - 1) / a.slices) + unit;
+    const size_t smem = (size_t)widest * sizeof(unsigned long long);
     cudaError_t e =
         cudaFuncSetAttribute(mix_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -238,5 +210,7 @@ cudaError_t launch_mix(const MixArgs& a, cudaStream_t stream)
     mix_kernel<<<grid, kMixThreads, smem, stream>>>(a);
     return cudaGetLastError();
 }
+
+int mix_min_slices(int vocab) { return (vocab + kMixMaxSliceTokens - 1) / kMixMaxSliceTokens; }
 
 }  // namespace nest

@@ -399,6 +399,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
         const int n = sh.cnt[qb];
         for (int j = lane; j < a.r; j += 32)
             out[(size_t)qb * a.r + j] = j < n ? cand[(size_t)qb * a.cap + j] : kNoCandidate;
+        if (lane == 0) a.cand_cnt[(size_t)item * NQ + qb] = n;
     }
 }
 

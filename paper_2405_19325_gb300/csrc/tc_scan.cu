@@ -268,6 +268,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int n = sh.cnt[b];
             for (int jj = e; jj < a.r; jj += kEpiThreads)
                 out[(size_t)b * a.r + jj] = jj < n ? cand[(size_t)b * a.cap + jj] : kNoCandidate;
+            if (e == 0) a.cand_cnt[(size_t)item * NQ + b] = n;
         }
     }
 
