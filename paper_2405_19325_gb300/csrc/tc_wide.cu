@@ -33,13 +33,13 @@ constexpr int kSelThreads = 1024;
 
 template <int NM>
 struct WideShared {
+    float qn[NM];      // ||q||^2 of the group's queries
+    uint32_t thr[NM];  // a key is admitted iff the fp32 bits of its distance are <= thr
     uint64_t full[kMaxStagesW];
     uint64_t empty[kMaxStagesW];
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
-    uint64_t thr[NM];
-    float qn[NM];
     uint32_t tmem_base;
     int abort;
     int issued;
@@ -61,6 +61,64 @@ __device__ __forceinline__ void wait_or_abort_w(uint64_t* bar, uint32_t parity, 
     if (!mbar_wait_bounded(bar, parity)) {
         record_status(status, NEST_ERR_TIMEOUT);
         *reinterpret_cast<volatile int*>(abort_flag) = 1;
+    }
+}
+
+// Epilogue of W accumulator columns (queries c0 .. c0 + W - 1) of one key
+// row: D = ||q||^2 + ||k||^2 - 2 q.k, clamped at 0, admitted at or below the
+// query's threshold.  The admission test is branch-free over the W columns.
+// When some lane admits a key, the warp forms each column's ballot, lane i
+// reserves room in column i's list with one atomic (all columns' atomics in
+// flight together), and every admitting lane writes its word.
+template <int W, int NM>
+__device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, int nqv, float kn,
+                                             bool valid, uint32_t key_idx, int lane,
+                                             const WideShared<NM>& sh, const WideArgs& a, int q0)
+{
+    uint32_t m = 0;
+#pragma unroll
+    for (int v = 0; v < W / 4; ++v) {
+        const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
+        const uint4 tv = *reinterpret_cast<const uint4*>(sh.thr + c0 + 4 * v);
+        const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
+        const uint32_t ta[4] = {tv.x, tv.y, tv.z, tv.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
+            dist = (dist <= 0.f) ? 0.f : dist;
+            m |= (__float_as_uint(dist) <= ta[k] ? 1u : 0u) << (4 * v + k);
+        }
+    }
+    // padding columns (no query) and rows past the range never append
+    const int ncol = nqv - c0;
+    const uint32_t colmask = ncol >= 32 ? ~0u : (ncol <= 0 ? 0u : (1u << ncol) - 1u);
+    m = valid ? (m & colmask) : 0u;
+    const uint32_t any = __reduce_or_sync(~0u, m);
+    if (any == 0) return;
+    uint32_t my_bal = 0;  // lane i: ballot of column c0 + i
+#pragma unroll
+    for (int i = 0; i < W; ++i) {
+        if ((any >> i) & 1u) {
+            const uint32_t bal = __ballot_sync(~0u, (m >> i) & 1u);
+            if (lane == i) my_bal = bal;
+        }
+    }
+    int base = 0;
+    if (my_bal != 0) base = atomicAdd(&a.cnt[q0 + c0 + lane], __popc(my_bal));
+    const uint32_t lt = lanemask_lt();
+#pragma unroll
+    for (int i = 0; i < W; ++i) {
+        if (!((any >> i) & 1u)) continue;
+        const int at = __shfl_sync(~0u, base, i);
+        const uint32_t bal = __shfl_sync(~0u, my_bal, i);
+        if ((m >> i) & 1u) {
+            float dist = fmaf(-2.f, __uint_as_float(acc[i]), sh.qn[c0 + i] + kn);
+            dist = (dist <= 0.f) ? 0.f : dist;
+            const uint64_t key = ((uint64_t)__float_as_uint(dist) << 32) | key_idx;
+            const long long pos = (long long)at + __popc(bal & lt);
+            if (pos < a.cap) a.cand[(int64_t)(q0 + c0 + i) * a.cap + pos] = key;
+            else record_status(a.status, NEST_ERR_OVERFLOW);
+        }
     }
 }
 
@@ -186,11 +244,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // distance of the sample (an upper bound of the true r-th distance),
         // or every key on the sampling pass itself (no s_sample).
         for (int j = e; j < NM; j += kEpiThreads) {
-            uint64_t thr = kNoCandidate;
+            uint32_t thr = 0xFFFFFFFFu;
             if (a.s_sample != nullptr && j < nqv) {
                 const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
-                if (s_r > -INFINITY)
-                    thr = ((uint64_t)__float_as_uint(-s_r) << 32) | 0xFFFFFFFFull;
+                if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
             }
             sh.thr[j] = thr;
         }
@@ -232,34 +289,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
             tc_fence_after();
             const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);
-#pragma unroll 1
-            for (int c0 = 0; c0 < NM; c0 += 16) {
+            const uint32_t key_idx = (uint32_t)(row * ks);
+            if constexpr (NM == 16) {
                 uint32_t acc[16];
-                tmem_ld_16(tbase + (uint32_t)c0, acc);
-                if (c0 + 16 == NM) {  // the whole accumulator has been read
-                    tc_fence_before();
-                    mbar_arrive(&sh.acc_empty[buf]);
-                }
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int col = c0 + i;
-                    float dist = fmaf(-2.f, __uint_as_float(acc[i]), sh.qn[col] + kn);
-                    dist = (dist <= 0.f) ? 0.f : dist;
-                    const uint64_t key =
-                        ((uint64_t)__float_as_uint(dist) << 32) | (uint32_t)(row * ks);
-                    // padding columns (no query) never append
-                    const bool accept = valid && col < nqv && key <= sh.thr[col];
-                    const uint32_t bal = __ballot_sync(~0u, accept);
-                    if (bal) {
-                        const int leader = __ffs(bal) - 1;
-                        long long at = 0;
-                        if (lane == leader) at = atomicAdd(&a.cnt[q0 + col], __popc(bal));
-                        at = __shfl_sync(~0u, at, leader);
-                        if (accept) {
-                            const long long pos = at + __popc(bal & lanemask_lt());
-                            if (pos < a.cap) a.cand[(int64_t)(q0 + col) * a.cap + pos] = key;
-                            else record_status(a.status, NEST_ERR_OVERFLOW);
+                tmem_ld_16(tbase, acc);
+                tc_fence_before();
+                mbar_arrive(&sh.acc_empty[buf]);
+                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, a, q0);
+            } else {
+                // two 32-column register buffers: the next TMEM load is in
+                // flight while the current columns are tested
+                uint32_t a0[32], a1[32];
+                tmem_ld_32_async(tbase, a0);
+#pragma unroll 1
+                for (int c0 = 0; c0 < NM; c0 += 64) {
+                    tmem_wait_ld(a0);
+                    if (c0 + 32 < NM) {
+                        tmem_ld_32_async(tbase + (uint32_t)(c0 + 32), a1);
+                    } else {
+                        tc_fence_before();
+                        mbar_arrive(&sh.acc_empty[buf]);
+                    }
+                    wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, a, q0);
+                    if (c0 + 32 < NM) {
+                        tmem_wait_ld(a1);
+                        if (c0 + 64 < NM) {
+                            tmem_ld_32_async(tbase + (uint32_t)(c0 + 64), a0);
+                        } else {
+                            tc_fence_before();
+                            mbar_arrive(&sh.acc_empty[buf]);
                         }
+                        wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, a, q0);
                     }
                 }
             }
