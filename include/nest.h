@@ -302,6 +302,8 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
  *   1  tensor-core scan with per-CTA top-r (bf16 keys, query groups of <= 16)
  *   2  tensor-core scan of large query batches against sampled admission
  *      thresholds (bf16 keys, more queries than one CTA keeps lists for)
+ *   3  the same with two 128-key tiles per pipeline stage (groups of 256
+ *      queries, when three 64 KiB stages fit in shared memory)
  * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
  */
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,

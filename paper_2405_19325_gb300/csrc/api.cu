@@ -808,7 +808,7 @@ int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r, int32
     SearchPlan sp;
     const nest_status_t st = plan_search(ds, B, r, ragged != 0, &sp);
     if (st != NEST_OK) return -(int32_t)st;
-    return sp.wide ? 2 : (sp.tc ? 1 : 0);
+    return sp.wide ? (sp.wpm.mb == 2 ? 3 : 2) : (sp.tc ? 1 : 0);
 }
 
 const char* nest_status_string(nest_status_t s)

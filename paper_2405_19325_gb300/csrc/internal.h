@@ -118,6 +118,7 @@ cudaError_t launch_tc_scan(const TcPlan& plan, const CUtensorMap& keys, const CU
 // Large query batches: threshold-admission scan into global lists + exact selection.
 struct WidePlan {
     int nm;       // MMA N = queries per CTA (16, 32, 64, 128 or 256)
+    int mb;       // 128-key tiles per pipeline stage (2 only for nm = 256)
     int stages;
     int groups;   // query groups of nm
     int parts;    // key-range parts (whole 128-key tiles)

@@ -122,6 +122,40 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
     }
 }
 
+// Drains one TMEM lane (this thread's key row) of an NM-column accumulator
+// at tbase, 32 columns per load with the next load in flight, and arrives
+// on `release` once the whole accumulator has been read.
+template <int NM>
+__device__ __forceinline__ void wide_drain_row(uint32_t tbase, uint64_t* release, int nqv, float kn,
+                                               bool valid, uint32_t key_idx, int lane,
+                                               const WideShared<NM>& sh, const WideArgs& a, int q0)
+{
+    static_assert(NM % 64 == 0 || NM == 32, "columns are drained in pairs of 32");
+    uint32_t a0[32], a1[32];
+    tmem_ld_32_async(tbase, a0);
+#pragma unroll 1
+    for (int c0 = 0; c0 < NM; c0 += 64) {
+        tmem_wait_ld(a0);
+        if (c0 + 32 < NM) {
+            tmem_ld_32_async(tbase + (uint32_t)(c0 + 32), a1);
+        } else {
+            tc_fence_before();
+            mbar_arrive(release);
+        }
+        wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, a, q0);
+        if (c0 + 32 < NM) {
+            tmem_wait_ld(a1);
+            if (c0 + 64 < NM) {
+                tmem_ld_32_async(tbase + (uint32_t)(c0 + 64), a0);
+            } else {
+                tc_fence_before();
+                mbar_arrive(release);
+            }
+            wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, a, q0);
+        }
+    }
+}
+
 template <int NM>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_wide_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
@@ -297,32 +331,191 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 mbar_arrive(&sh.acc_empty[buf]);
                 wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, a, q0);
             } else {
-                // two 32-column register buffers: the next TMEM load is in
-                // flight while the current columns are tested
-                uint32_t a0[32], a1[32];
-                tmem_ld_32_async(tbase, a0);
-#pragma unroll 1
-                for (int c0 = 0; c0 < NM; c0 += 64) {
-                    tmem_wait_ld(a0);
-                    if (c0 + 32 < NM) {
-                        tmem_ld_32_async(tbase + (uint32_t)(c0 + 32), a1);
-                    } else {
-                        tc_fence_before();
-                        mbar_arrive(&sh.acc_empty[buf]);
+                wide_drain_row<NM>(tbase, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane, sh, a, q0);
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kCols);
+    }
+    if (tid == 0 && *reinterpret_cast<volatile int*>(&sh.abort)) {
+        const int issued = *reinterpret_cast<volatile int*>(&sh.issued);
+        for (int s = max(0, issued - a.stages); s < issued; ++s)
+            (void)mbar_wait_bounded(&sh.full[s % a.stages], (uint32_t)(s / a.stages) & 1u);
+    }
+}
+
+// Two 128-key tiles per pipeline stage for groups of 256 queries: both
+// tiles' MMAs (M = 128, N = 256, K = 16 each) read the stage's query chunk,
+// so one 64 KiB stage (32 KiB of keys, 32 KiB of queries) carries twice the
+// MMA work of a one-tile stage and the stage ring covers twice the latency.
+// The two 256-column fp32 accumulators fill TMEM, so a tile pair's epilogue
+// runs between its last MMA and the next pair's first; eight epilogue warps
+// (two per TMEM lane quarter, one per tile) keep that gap short.
+constexpr int kWide2Threads = 64 + 2 * kEpiThreads;
+
+__global__ void __launch_bounds__(kWide2Threads, 1)
+    tc_wide2_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
+                    const WideArgs a)
+{
+    constexpr int NM = 256;
+    constexpr int kStage = 2 * kABytes + NM * kChunkK * 2;
+    constexpr uint32_t kCols = 512;
+    constexpr int kPairKeys = 2 * kTileM;
+
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    unsigned char* stages = smem;
+    WideShared<NM>& sh = *reinterpret_cast<WideShared<NM>*>(smem + (size_t)a.stages * kStage);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int part = blockIdx.x / a.groups, group = blockIdx.x - part * a.groups;
+    const int q0 = group * NM;
+    const int nqv = min(NM, a.B - q0);
+
+    const int64_t pairs = (a.N + kPairKeys - 1) / kPairKeys;
+    const int64_t t0 = pairs * part / a.parts, t1 = pairs * (part + 1) / a.parts;
+    const int64_t lo = t0 * kPairKeys;
+    const int64_t hi = min(a.N, t1 * kPairKeys);
+    const int npairs = (int)(t1 - t0);
+    const int kc = a.kchunks;
+    const int nsteps = npairs * kc;
+
+    if (tid == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&sh.full[s], 1);
+            mbar_init(&sh.empty[s], 1);
+        }
+        mbar_init(&sh.acc_full[0], 1);
+        mbar_init(&sh.acc_empty[0], 2 * kEpiThreads);
+        mbar_init(&sh.drain, 1);
+        sh.abort = 0;
+        sh.issued = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) tmem_alloc(&sh.tmem_base, kCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0 && nsteps > 0) {
+            const uint64_t policy = l2_policy_evict_first();
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int s = 0; s < nsteps; ++s) {
+                const int t = s / kc, c = s - t * kc;
+                if (s >= a.stages) {
+                    wait_or_abort_w(&sh.empty[slot], phase ^ 1u, &sh.abort, a.status);
+                    if (*reinterpret_cast<volatile int*>(&sh.abort)) break;
+                }
+                unsigned char* st = stages + (size_t)slot * kStage;
+                mbar_arrive_expect_tx(&sh.full[slot], kStage);
+                const int32_t y = (int32_t)(lo + (int64_t)t * kPairKeys);
+                if (group == a.groups - 1) {
+                    tma_load_2d_hint(st, &tmK, c * kChunkK, y, &sh.full[slot], policy);
+                    tma_load_2d_hint(st + kABytes, &tmK, c * kChunkK, y + kTileM, &sh.full[slot],
+                                     policy);
+                } else {
+                    tma_load_2d(st, &tmK, c * kChunkK, y, &sh.full[slot]);
+                    tma_load_2d(st + kABytes, &tmK, c * kChunkK, y + kTileM, &sh.full[slot]);
+                }
+                tma_load_2d(st + 2 * kABytes, &tmQ, c * kChunkK, q0, &sh.full[slot]);
+                *reinterpret_cast<volatile int*>(&sh.issued) = s + 1;
+                if (++slot == a.stages) {
+                    slot = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && nsteps > 0) {
+            constexpr uint32_t idesc = mma_idesc_bf16(kTileM, NM);
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int j = 0; j < npairs; ++j) {
+                if (j >= 1)
+                    wait_or_abort_w(&sh.acc_empty[0], (uint32_t)(j - 1) & 1u, &sh.abort, a.status);
+                tc_fence_after();
+                for (int c = 0; c < kc; ++c) {
+                    wait_or_abort_w(&sh.full[slot], phase, &sh.abort, a.status);
+                    tc_fence_after();
+                    const unsigned char* st = stages + (size_t)slot * kStage;
+                    const uint64_t ad0 = smem_desc_sw128(st);
+                    const uint64_t ad1 = smem_desc_sw128(st + kABytes);
+                    const uint64_t bd = smem_desc_sw128(st + 2 * kABytes);
+#pragma unroll
+                    for (int k = 0; k < kChunkK / 16; ++k) {
+                        mma_bf16(tmem, ad0 + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
+                        mma_bf16(tmem + (uint32_t)NM, ad1 + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
                     }
-                    wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, a, q0);
-                    if (c0 + 32 < NM) {
-                        tmem_wait_ld(a1);
-                        if (c0 + 64 < NM) {
-                            tmem_ld_32_async(tbase + (uint32_t)(c0 + 64), a0);
-                        } else {
-                            tc_fence_before();
-                            mbar_arrive(&sh.acc_empty[buf]);
-                        }
-                        wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, a, q0);
+                    mma_commit(&sh.empty[slot]);
+                    if (++slot == a.stages) {
+                        slot = 0;
+                        phase ^= 1u;
+                    }
+                }
+                mma_commit(&sh.acc_full[0]);
+            }
+            mma_commit(&sh.drain);
+            (void)mbar_wait_bounded(&sh.drain, 0);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int e = tid - 64;  // 0 .. 255
+        const int quarter = warp & 3;
+        const int h = (warp - 2) >> 2;  // key tile of the pair this warp drains
+        for (int j = e; j < NM; j += 2 * kEpiThreads) {
+            uint32_t thr = 0xFFFFFFFFu;
+            if (a.s_sample != nullptr && j < nqv) {
+                const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+            }
+            sh.thr[j] = thr;
+        }
+        const unsigned char* qb = static_cast<const unsigned char*>(a.q);
+        const int chunks = a.d / 8;
+        for (int j = warp - 2; j < NM; j += 8) {
+            float s = 0.f;
+            if (j < nqv) {
+                const unsigned char* row = qb + (size_t)(q0 + j) * a.d * 2;
+                for (int c = lane; c < chunks; c += 32) {
+                    const uint4 v = ld_global_nc_v4(row + (size_t)c * 16);
+                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float lo_ = __uint_as_float(w[i] << 16);
+                        const float hi_ = __uint_as_float(w[i] & 0xffff0000u);
+                        s = fmaf(lo_, lo_, s);
+                        s = fmaf(hi_, hi_, s);
                     }
                 }
             }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
+            if (lane == 0) sh.qn[j] = s;
+        }
+        named_barrier(2, 2 * kEpiThreads);
+
+        const int64_t ks = a.key_stride;
+        const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM);
+        for (int j = 0; j < npairs; ++j) {
+            const int64_t row = lo + (int64_t)j * kPairKeys + h * kTileM + 32 * quarter + lane;
+            const float kn = row < hi ? __ldg(a.knorm + row * ks) : 0.f;
+            const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
+            wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
+            tc_fence_after();
+            wide_drain_row<NM>(tbase, &sh.acc_empty[0], nqv, kn, valid, (uint32_t)(row * ks), lane,
+                               sh, a, q0);
         }
     }
 
@@ -406,11 +599,25 @@ template <int NM>
 bool wide_plan_nm(size_t smem_limit, WidePlan* p)
 {
     const size_t fixed = wide_fixed<NM>();
+    if (NM == 256) {
+        // two key tiles per stage when three 64 KiB stages fit
+        const size_t st2 = (size_t)(2 * kABytes + NM * kChunkK * 2);
+        if (fixed + 3 * st2 <= smem_limit) {
+            int stages = (int)((smem_limit - fixed) / st2);
+            stages = stages > kMaxStagesW ? kMaxStagesW : stages;
+            p->nm = NM;
+            p->mb = 2;
+            p->stages = stages;
+            p->smem = fixed + (size_t)stages * st2;
+            return true;
+        }
+    }
     const size_t st = (size_t)stage_bytes<NM>();
     if (fixed + 3 * st > smem_limit) return false;
     int stages = (int)((smem_limit - fixed) / st);
     stages = stages > kMaxStagesW ? kMaxStagesW : stages;
     p->nm = NM;
+    p->mb = 1;
     p->stages = stages;
     p->smem = fixed + (size_t)stages * st;
     return true;
@@ -420,6 +627,13 @@ template <int NM>
 cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
                            const WideArgs& a, cudaStream_t stream)
 {
+    if (NM == 256 && p.mb == 2) {
+        cudaError_t e = cudaFuncSetAttribute(tc_wide2_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+        if (e != cudaSuccess) return e;
+        tc_wide2_kernel<<<p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ, a);
+        return cudaGetLastError();
+    }
     auto kern = tc_wide_kernel<NM>;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);

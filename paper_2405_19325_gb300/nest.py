@@ -350,7 +350,8 @@ class Datastore:
     def launch_count(self) -> int:
         return int(self._lib.nest_launch_count(self._h))
 
-    SEARCH_PATHS = {0: "scan_topr_kernel", 1: "tc_scan_kernel", 2: "tc_wide_kernel"}
+    SEARCH_PATHS = {0: "scan_topr_kernel", 1: "tc_scan_kernel", 2: "tc_wide_kernel",
+                    3: "tc_wide2_kernel"}
 
     def search_path(self, B: int, r: int, ragged: bool = False) -> str:
         """Name of the distance-scan kernel a search of this shape runs."""

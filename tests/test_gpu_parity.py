@@ -319,6 +319,23 @@ def test_wide_batch_single_pass_over_300_queries(nest):
     run_and_check(nest, K, V, q, p_lm, 64, 1 / np.sqrt(128), 0.8, 500, "bf16")
 
 
+@pytest.mark.parametrize("N,d,B,r", [
+    (200036, 200, 260, 64),   # two passes; last pair: one partial tile, one tile past N
+    (70017, 64, 256, 33),     # single pass, one full group, d = one K chunk, 1-row tile
+])
+def test_two_tile_wide_kernel_edges(nest, N, d, B, r):
+    """Groups of 256 queries run two 128-key tiles per pipeline stage: a
+    partial last group (padding columns), d not a multiple of 64 (the last
+    K chunk half outside the rows), and a last tile pair whose second tile
+    lies wholly past the last key."""
+    K, V, q, p_lm = _random_case(N, d, B, 900, "bf16", seed=23 + d, centres=48)
+    ds = nest.Datastore(K.cuda(), V.cuda(), 900)
+    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.close()
+    rows = list(range(0, B, 7)) + [B - 1]
+    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 900, "bf16", check_rows=rows)
+
+
 def test_large_batch_shape_sampled_rows(nest):
     """Large-batch shape: bf16 d=4096, B=512, r=256, clustered keys (N reduced
     to 524,288); the oracle checks 12 query rows spread over the batch."""
