@@ -289,11 +289,20 @@ def run_reference(args, w, world, rank):
 # Only valid for that kernel version on the default decode workload.
 DECODE_TC_SCAN_TRAFFIC = 537.27e6 * 16 + 3.05e6
 
+# Same for the large-batch main pass, from profiles/tc_wide2_large_batch_B512.md:
+# the 262,144-key case scaled by 16 to the default 4,194,304 keys (key reads
+# and, with the sample size fixed at 65,536 keys, survivor writes both grow
+# with N).  Only valid for that kernel version on the default large batch.
+LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.316181e9 + 6.842624e6) * 16
+
 
 def dram_traffic(w, args, kernel):
-    if (w.name == "decode" and kernel == "tc_scan_kernel" and args.N is None
-            and args.B is None):
+    if args.N is not None or args.B is not None:
+        return None
+    if w.name == "decode" and kernel == "tc_scan_kernel":
         return DECODE_TC_SCAN_TRAFFIC
+    if w.name == "large_batch" and kernel == "tc_wide2_kernel":
+        return LARGE_BATCH_TC_WIDE2_TRAFFIC
     return None
 
 
