@@ -293,6 +293,26 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
 
 // Large query batches: [sample pass, selection of the sample,] thresholded
 // pass over all keys, exact selection of the survivors.
+// List slots each epilogue warp of the main pass reserves per query at a
+// time.  About a fraction r / sample_rows of the keys pass the sample's r-th
+// distance, so a warp that drains `rows` key rows admits about
+// rows * r / sample_rows keys per query; it reserves twice that plus 16,
+// limited so that the first blocks of all warps leave room for twice the
+// expected survivors in the list.  Below 8 slots it is not worth it (0: one
+// atomic per admitting column).
+int32_t wide_reservation(const SearchPlan& sp, int64_t N, int32_t r)
+{
+    const int epi_warps = sp.wpm.mb == 2 ? 8 : 4;
+    const int64_t unit = (int64_t)kTcTileKeys * sp.wpm.mb;
+    const int64_t units = (N + unit - 1) / unit;
+    const int64_t rows = (units + sp.wpm.parts - 1) / sp.wpm.parts * 32;
+    const int64_t per_warp = (rows * r + sp.sample_rows - 1) / sp.sample_rows;
+    const int64_t expect = (N * r + sp.sample_rows - 1) / sp.sample_rows;
+    const int64_t room = (sp.cap_m - 2 * expect) / ((int64_t)sp.wpm.parts * epi_warps);
+    const int64_t R = std::min<int64_t>(2 * per_warp + 16, room);
+    return R >= 8 ? (int32_t)std::min<int64_t>(R, 1 << 20) : 0;
+}
+
 nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* q, int32_t B,
                           int32_t r, const uint32_t* key_mask, float* s_out, int64_t* idx_out,
                           uint64_t* scratch, bool timed, cudaStream_t stream)
@@ -374,6 +394,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     wa.N = ds->N;
     wa.parts = sp.wpm.parts;
     wa.key_stride = 1;
+    wa.resv = wide_reservation(sp, ds->N, r);
     if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
     e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
     if (e != cudaSuccess) return from_cuda(e);

@@ -143,6 +143,10 @@ struct WideArgs {
     int32_t stages;
     int32_t kchunks;
     int64_t key_stride;  // row i of the key tensor map is key i * key_stride
+    // > 0: each epilogue warp reserves list slots per query in blocks of
+    // resv (one atomic per block) and pads unused slots with kNoCandidate,
+    // so cnt counts reserved slots.  0: one atomic per admitting column.
+    int32_t resv;
 };
 
 struct GselectArgs {

@@ -260,4 +260,13 @@ __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32])
                  : "memory");
 }
 
+// Stores v to shared memory at p when pred holds, without a branch.
+__device__ __forceinline__ void st_shared_u32_if(bool pred, const uint32_t* p, uint32_t v)
+{
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t@q st.shared.u32 [%1], %2;\n\t}" ::"r"(
+            (int)pred),
+        "r"(smem_addr(p)), "r"(v));
+}
+
 }  // namespace nest

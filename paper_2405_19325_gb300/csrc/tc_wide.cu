@@ -31,10 +31,20 @@ constexpr int kMaxStagesW = 12;
 constexpr int kEpiThreads = 128;
 constexpr int kSelThreads = 1024;
 
+constexpr int kMaxEpiWarps = 8;
+constexpr int kStageK = 4;  // admitted keys a lane stages per 32-column block
+
 template <int NM>
 struct WideShared {
     float qn[NM];      // ||q||^2 of the group's queries
     uint32_t thr[NM];  // a key is admitted iff the fp32 bits of its distance are <= thr
+    // Slots [x, y) of query column c's global list reserved by epilogue warp
+    // w and not yet written (used when WideArgs::resv > 0); x passes y once
+    // the block is used up.
+    int2 resv[kMaxEpiWarps][NM];
+    // Distance bits of the keys a lane admitted in one 32-column block, in
+    // column order: [warp][k][lane].
+    uint32_t stage[kMaxEpiWarps][kStageK][32];
     uint64_t full[kMaxStagesW];
     uint64_t empty[kMaxStagesW];
     uint64_t acc_full[2];
@@ -64,16 +74,33 @@ __device__ __forceinline__ void wait_or_abort_w(uint64_t* bar, uint32_t parity, 
     }
 }
 
+// Pads slots [from, to) of list `col` with kNoCandidate (reserved, never written).
+__device__ __forceinline__ void wide_pad(const WideArgs& a, int64_t col, int from, int to)
+{
+    uint64_t* list = a.cand + col * a.cap;
+    const int end = to < a.cap ? to : (int)a.cap;
+    for (int p = from; p < end; ++p) list[p] = kNoCandidate;
+}
+
 // Epilogue of W accumulator columns (queries c0 .. c0 + W - 1) of one key
 // row: D = ||q||^2 + ||k||^2 - 2 q.k, clamped at 0, admitted at or below the
 // query's threshold.  The admission test is branch-free over the W columns.
-// When some lane admits a key, the warp forms each column's ballot, lane i
-// reserves room in column i's list with one atomic (all columns' atomics in
-// flight together), and every admitting lane writes its word.
+//
+// Appending, when some lane admits a key:
+//  * with reservations (a.resv > 0) and at most kStageK admitted keys per
+//    lane, a branch-free pass stages each lane's admitted distances in
+//    shared memory, then each lane takes a slot per key from this warp's
+//    block for that column (a shared-memory atomic), or one fresh slot of
+//    the list once the block is used up;
+//  * otherwise the warp forms each column's ballot, lane i takes room in
+//    column i's list (from the warp's block, or with one global atomic; all
+//    columns' atomics in flight together), and every admitting lane writes
+//    its word.
 template <int W, int NM>
 __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, int nqv, float kn,
                                              bool valid, uint32_t key_idx, int lane,
-                                             const WideShared<NM>& sh, const WideArgs& a, int q0)
+                                             const WideShared<NM>& sh, int2* resv,
+                                             uint32_t* stage, const WideArgs& a, int q0)
 {
     uint32_t m = 0;
 #pragma unroll
@@ -95,6 +122,38 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
     m = valid ? (m & colmask) : 0u;
     const uint32_t any = __reduce_or_sync(~0u, m);
     if (any == 0) return;
+    if (a.resv > 0 && __all_sync(~0u, __popc(m) <= kStageK)) {
+        uint32_t* st = stage + lane;
+        int n = 0;
+#pragma unroll
+        for (int v = 0; v < W / 4; ++v) {
+            const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
+            const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
+                dist = (dist <= 0.f) ? 0.f : dist;
+                const int b = (m >> (4 * v + k)) & 1u;
+                st_shared_u32_if(b != 0, st + n * 32, __float_as_uint(dist));
+                n += b;
+            }
+        }
+        __syncwarp();
+        uint32_t mm = m;
+        for (int j = 0; j < n; ++j) {
+            const int col = c0 + __ffs(mm) - 1;
+            mm &= mm - 1;
+            const uint32_t dbits = st[j * 32];
+            int pos = atomicAdd(&resv[col].x, 1);
+            if (pos >= resv[col].y) pos = atomicAdd(&a.cnt[q0 + col], 1);
+            if (pos < a.cap)
+                a.cand[(int64_t)(q0 + col) * a.cap + pos] = ((uint64_t)dbits << 32) | key_idx;
+            else
+                record_status(a.status, NEST_ERR_OVERFLOW);
+        }
+        __syncwarp();
+        return;
+    }
     uint32_t my_bal = 0;  // lane i: ballot of column c0 + i
 #pragma unroll
     for (int i = 0; i < W; ++i) {
@@ -104,7 +163,25 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
         }
     }
     int base = 0;
-    if (my_bal != 0) base = atomicAdd(&a.cnt[q0 + c0 + lane], __popc(my_bal));
+    if (my_bal != 0) {
+        const int need = __popc(my_bal);
+        if (a.resv > 0) {
+            // from this warp's block for the column; a new block (padding the
+            // rest of the old one) when it cannot hold them
+            int2 rv = resv[c0 + lane];
+            if (rv.x + need > rv.y) {
+                wide_pad(a, q0 + c0 + lane, rv.x, rv.y);
+                const int blk = need > a.resv ? need : a.resv;
+                rv.x = atomicAdd(&a.cnt[q0 + c0 + lane], blk);
+                rv.y = rv.x + blk;
+            }
+            base = rv.x;
+            rv.x += need;
+            resv[c0 + lane] = rv;
+        } else {
+            base = atomicAdd(&a.cnt[q0 + c0 + lane], need);
+        }
+    }
     const uint32_t lt = lanemask_lt();
 #pragma unroll
     for (int i = 0; i < W; ++i) {
@@ -122,13 +199,44 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
     }
 }
 
+// First reservations: lane i reserves a.resv slots in each column i + 32k of
+// the group for this warp (its atomics all in flight together).
+template <int NM>
+__device__ __forceinline__ void wide_reserve(int2* resv, int nqv, int lane, const WideArgs& a,
+                                             int q0)
+{
+    for (int c = lane; c < NM; c += 32) {
+        int2 rv = make_int2(0, 0);
+        if (a.resv > 0 && c < nqv) {
+            rv.x = atomicAdd(&a.cnt[q0 + c], a.resv);
+            rv.y = rv.x + a.resv;
+        }
+        resv[c] = rv;
+    }
+    __syncwarp();
+}
+
+// Pads what is left of this warp's blocks once the pass is done.
+template <int NM>
+__device__ __forceinline__ void wide_release(const int2* resv, int nqv, int lane, const WideArgs& a,
+                                             int q0)
+{
+    if (a.resv <= 0) return;
+    __syncwarp();
+    for (int c = lane; c < nqv && c < NM; c += 32) {
+        const int2 rv = resv[c];
+        if (rv.x < rv.y) wide_pad(a, q0 + c, rv.x, rv.y);
+    }
+}
+
 // Drains one TMEM lane (this thread's key row) of an NM-column accumulator
 // at tbase, 32 columns per load with the next load in flight, and arrives
 // on `release` once the whole accumulator has been read.
 template <int NM>
 __device__ __forceinline__ void wide_drain_row(uint32_t tbase, uint64_t* release, int nqv, float kn,
                                                bool valid, uint32_t key_idx, int lane,
-                                               const WideShared<NM>& sh, const WideArgs& a, int q0)
+                                               const WideShared<NM>& sh, int2* resv,
+                                               uint32_t* stage, const WideArgs& a, int q0)
 {
     static_assert(NM % 64 == 0 || NM == 32, "columns are drained in pairs of 32");
     uint32_t a0[32], a1[32];
@@ -142,7 +250,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, uint64_t* release
             tc_fence_before();
             mbar_arrive(release);
         }
-        wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, a, q0);
+        wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a, q0);
         if (c0 + 32 < NM) {
             tmem_wait_ld(a1);
             if (c0 + 64 < NM) {
@@ -151,7 +259,8 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, uint64_t* release
                 tc_fence_before();
                 mbar_arrive(release);
             }
-            wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, a, q0);
+            wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, resv, stage, a,
+                                    q0);
         }
     }
 }
@@ -309,6 +418,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (lane == 0) sh.qn[j] = s;
         }
         named_barrier(2, kEpiThreads);
+        int2* resv = sh.resv[warp - 2];
+        uint32_t* stage = &sh.stage[warp - 2][0][0];
+        wide_reserve<NM>(resv, nqv, lane, a, q0);
 
         const int row_in_tile = 32 * quarter + lane;
         const int64_t ks = a.key_stride;  // row i of the tensor map is key i * ks
@@ -329,11 +441,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tmem_ld_16(tbase, acc);
                 tc_fence_before();
                 mbar_arrive(&sh.acc_empty[buf]);
-                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, a, q0);
+                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a, q0);
             } else {
-                wide_drain_row<NM>(tbase, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane, sh, a, q0);
+                wide_drain_row<NM>(tbase, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane, sh,
+                                   resv, stage, a, q0);
             }
         }
+        wide_release<NM>(resv, nqv, lane, a, q0);
     }
 
     tc_fence_before();
@@ -505,6 +619,9 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             if (lane == 0) sh.qn[j] = s;
         }
         named_barrier(2, 2 * kEpiThreads);
+        int2* resv = sh.resv[warp - 2];
+        uint32_t* stage = &sh.stage[warp - 2][0][0];
+        wide_reserve<NM>(resv, nqv, lane, a, q0);
 
         const int64_t ks = a.key_stride;
         const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM);
@@ -515,8 +632,9 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
             tc_fence_after();
             wide_drain_row<NM>(tbase, &sh.acc_empty[0], nqv, kn, valid, (uint32_t)(row * ks), lane,
-                               sh, a, q0);
+                               sh, resv, stage, a, q0);
         }
+        wide_release<NM>(resv, nqv, lane, a, q0);
     }
 
     tc_fence_before();
@@ -578,8 +696,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
     float* so = a.s_out + (int64_t)q * a.r;
     int64_t* io = a.idx_out + (int64_t)q * a.r;
     for (int j = tid; j < a.r; j += kSelThreads) {
-        if (j < n) {
-            const uint64_t e = sort_buf[j];
+        const uint64_t e = j < n ? sort_buf[j] : kNoCandidate;
+        if (e != kNoCandidate) {  // reserved slots never written hold kNoCandidate
             so[j] = -__uint_as_float((uint32_t)(e >> 32));
             io[j] = (int64_t)(uint32_t)e;
         } else {
