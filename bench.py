@@ -293,7 +293,7 @@ DECODE_TC_SCAN_TRAFFIC = 537.27e6 * 16 + 3.05e6
 # the 262,144-key case scaled by 16 to the default 4,194,304 keys (key reads
 # and, with the sample size fixed at 65,536 keys, survivor writes both grow
 # with N).  Only valid for that kernel version on the default large batch.
-LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.316181e9 + 6.842624e6) * 16
+LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.339577e9 + 22.096384e6) * 16
 
 
 def dram_traffic(w, args, kernel):
