@@ -115,22 +115,7 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
         const int P2 = next_pow2(n > 0 ? n : 1);
         for (int j = n + tid; j < P2; j += kMergeThreads) buf[j] = kNoCandidate;
         __syncthreads();
-        for (int k = 2; k <= P2; k <<= 1) {
-            for (int jj = k >> 1; jj > 0; jj >>= 1) {
-                for (int i = tid; i < P2; i += kMergeThreads) {
-                    const int l = i ^ jj;
-                    if (l > i) {
-                        const uint64_t x = buf[i], y = buf[l];
-                        const bool ascending = (i & k) == 0;
-                        if ((x > y) == ascending) {
-                            buf[i] = y;
-                            buf[l] = x;
-                        }
-                    }
-                }
-                __syncthreads();
-            }
-        }
+        bitonic_sort<kMergeThreads>(buf, P2, tid, [] { __syncthreads(); });
         float* so = a.s_out + (int64_t)b * a.r;
         int64_t* io = a.idx_out + (int64_t)b * a.r;
         for (int j = tid; j < a.r; j += kMergeThreads) {

@@ -678,21 +678,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
     while (P2 < (n > 0 ? n : 1)) P2 <<= 1;
     for (int j = tid; j < P2; j += kSelThreads) sort_buf[j] = j < n ? list[j] : kNoCandidate;
     __syncthreads();
-    for (int k = 2; k <= P2; k <<= 1) {
-        for (int jj = k >> 1; jj > 0; jj >>= 1) {
-            for (int i = tid; i < P2; i += kSelThreads) {
-                const int l = i ^ jj;
-                if (l > i) {
-                    const uint64_t x = sort_buf[i], y = sort_buf[l];
-                    if ((x > y) == ((i & k) == 0)) {
-                        sort_buf[i] = y;
-                        sort_buf[l] = x;
-                    }
-                }
-            }
-            __syncthreads();
-        }
-    }
+    bitonic_sort<kSelThreads>(sort_buf, P2, tid, [] { __syncthreads(); });
     float* so = a.s_out + (int64_t)q * a.r;
     int64_t* io = a.idx_out + (int64_t)q * a.r;
     for (int j = tid; j < a.r; j += kSelThreads) {
