@@ -148,7 +148,7 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
         sp->parts = p.parts;
     }
     sp->cand_words = (size_t)sp->groups * sp->parts * sp->nq * r;
-    const int per = merge_lists_per_cta(r);
+    const int per = merge_fanin(sp->parts, r);
     const int lvl1 = (sp->parts + per - 1) / per;
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
     // int32 counts: [groups * parts * nq] then [B * lvl1], as 64-bit words
@@ -490,7 +490,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
     ma.idx_out = idx_out;
     bool into_b = true;
     for (;;) {
-        ma.per_cta = std::min(merge_lists_per_cta(r), ma.lists);
+        ma.per_cta = merge_fanin(ma.lists, r);
         const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
         const bool last = groups == 1;
         ma.out = into_b ? regionB : regionA;

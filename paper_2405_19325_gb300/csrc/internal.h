@@ -183,6 +183,8 @@ struct MergeArgs {
 };
 
 int merge_lists_per_cta(int r);
+// Lists one merge CTA takes at a level with `lists` input lists per query.
+int merge_fanin(int lists, int r);
 size_t merge_smem_bytes(int per_cta, int r);
 cudaError_t launch_merge(const MergeArgs& args, bool last, cudaStream_t stream);
 

@@ -75,29 +75,26 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
     __syncthreads();
     const int total = sh.off[nl];
 
-    // copy the real entries: entry e of the concatenation belongs to the list
-    // whose offset range holds it (binary search over the offsets)
-    for (int e0 = tid; e0 < total; e0 += 4 * kMergeThreads) {
-        uint64_t v[4];
-        int at[4];
+    // copy the real entries: warp w copies lists w, w + 32, ... to their
+    // offsets, eight loads in flight per lane
+    for (int l = warp; l < nl; l += kMergeThreads / 32) {
+        const int o = sh.off[l], len = sh.off[l + 1] - o;
+        const uint64_t* ls = src + (int64_t)(l0 + l) * a.list_stride;
+        for (int j0 = lane; j0 < len; j0 += 8 * 32) {
+            uint64_t v[8];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int e = e0 + u * kMergeThreads;
-            at[u] = e;
-            if (e < total) {
-                int lo = 0, hi = nl;  // find the last l with off[l] <= e
-                while (hi - lo > 1) {
-                    const int mid = (lo + hi) >> 1;
-                    if (sh.off[mid] <= e) lo = mid;
-                    else hi = mid;
-                }
-                v[u] = src[(int64_t)(l0 + lo) * a.list_stride + (e - sh.off[lo])];
+            for (int u = 0; u < 8; ++u) {
+                const int j = j0 + 32 * u;
+                if (j < len) v[u] = ls[j];
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int j = j0 + 32 * u;
+                if (j < len) buf[o + j] = v[u];
             }
         }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-            if (at[u] < total) buf[at[u]] = v[u];
     }
+    __syncthreads();
     if (tid == 0) {
         sh.cnt = total;
         sh.thr = kNoCandidate;
@@ -138,6 +135,19 @@ int merge_lists_per_cta(int r)
     int per = (int)(kMergeBufBytes / ((size_t)r * 8));
     per = per > kMaxListsPerCta ? kMaxListsPerCta : per;
     return per < 2 ? 2 : per;
+}
+
+int merge_fanin(int lists, int r)
+{
+    const int maxper = merge_lists_per_cta(r);
+    if (lists <= maxper) return lists;
+    // about sqrt(lists) per CTA balances two levels, but no fewer than the
+    // next level needs to fit one CTA
+    int per = 1;
+    while (per * per < lists) ++per;
+    const int need = (lists + maxper - 1) / maxper;
+    per = per > need ? per : need;
+    return per < maxper ? per : maxper;
 }
 
 size_t merge_smem_bytes(int per_cta, int r)
