@@ -210,6 +210,29 @@ NEST_API nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_
                             void* stream);
 
 /*
+ * nest_knn_step from host memory: the query batch, the segment offsets (or
+ * NULL) and p_LM are copied to device buffers the handle owns, the step runs
+ * on `stream`, and p_M, s and idx are copied back; the call returns once
+ * `stream` has finished (or with the first error).  Same arguments as
+ * nest_knn_step except that every pointer is a host pointer (page-locked
+ * memory lets the copies run asynchronously; pageable memory works but the
+ * driver stages it) and no p_kNN is returned.
+ *
+ * p_LM goes in, and s and idx come back, on a side stream the handle owns
+ * (ordered with `stream` by events), so those copies overlap the search and
+ * the mix.  The device buffers grow on demand with cudaMalloc, the side
+ * stream is created on the first call, and nest_datastore_destroy frees
+ * both; calls on one handle must not overlap.  Device-side
+ * errors of the kernels are reported by nest_device_status, as for
+ * nest_knn_step.  The paper's method is the same as nest_knn_step (Eq. 1-3);
+ * only the data movement differs.
+ */
+NEST_API nest_status_t nest_knn_step_host(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                                          const int64_t* seg_off, const float* p_lm, float mu,
+                                          float lambda, float* s_out, int64_t* idx_out,
+                                          float* p_m_out, void* stream);
+
+/*
  * nest_knn_search over the keys not yet used in this generation: accepted
  * spans are masked out of the datastore and never retrieved again
  * (Sec. 3.4, last paragraph).

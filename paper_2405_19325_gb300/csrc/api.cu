@@ -29,6 +29,10 @@ struct nest_datastore {
     int* status = nullptr;   // owned: device status word
     uint64_t* scratch = nullptr;  // owned: candidate lists of the search
     size_t scratch_words = 0;
+    unsigned char* host_stage = nullptr;  // owned: device copies for nest_knn_step_host
+    size_t host_stage_bytes = 0;
+    cudaStream_t aux = nullptr;           // owned: side stream of nest_knn_step_host
+    cudaEvent_t aux_ev[3] = {nullptr, nullptr, nullptr};
     bool timing = false;
     std::vector<cudaEvent_t> events;  // pairs (start, end)
     size_t events_used = 0;
@@ -258,6 +262,48 @@ nest_status_t record_event(nest_datastore* ds, cudaStream_t stream)
 }
 
 // Device pointers only: plain host memory would fault on GPUs that cannot reach it.
+// Device buffers of nest_knn_step_host, grown on demand (never shrunk).
+nest_status_t ensure_host_stage(nest_datastore* ds, size_t bytes)
+{
+    if (bytes <= ds->host_stage_bytes) return NEST_OK;
+    if (ds->host_stage) {
+        cudaError_t e = cudaFree(ds->host_stage);
+        ds->host_stage = nullptr;
+        ds->host_stage_bytes = 0;
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    void* p = nullptr;
+    cudaError_t e = cudaMalloc(&p, bytes);
+    if (e != cudaSuccess) {
+        (void)cudaGetLastError();
+        return NEST_ERR_OOM;
+    }
+    ds->host_stage = static_cast<unsigned char*>(p);
+    ds->host_stage_bytes = bytes;
+    return NEST_OK;
+}
+
+size_t round256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// The side stream and events of nest_knn_step_host, created on first use.
+nest_status_t ensure_aux(nest_datastore* ds)
+{
+    if (ds->aux) return NEST_OK;
+    cudaError_t e = cudaStreamCreateWithFlags(&ds->aux, cudaStreamNonBlocking);
+    for (int i = 0; i < 3 && e == cudaSuccess; ++i)
+        e = cudaEventCreateWithFlags(&ds->aux_ev[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        for (cudaEvent_t& ev : ds->aux_ev) {
+            if (ev) (void)cudaEventDestroy(ev);
+            ev = nullptr;
+        }
+        if (ds->aux) (void)cudaStreamDestroy(ds->aux);
+        ds->aux = nullptr;
+        return from_cuda(e);
+    }
+    return NEST_OK;
+}
+
 bool is_device_pointer(const void* p)
 {
     cudaPointerAttributes at;
@@ -626,6 +672,10 @@ nest_status_t nest_datastore_destroy(nest_datastore_t* ds)
     if (ds->knorm) keep(cudaFree(ds->knorm));
     if (ds->status) keep(cudaFree(ds->status));
     if (ds->scratch) keep(cudaFree(ds->scratch));
+    if (ds->host_stage) keep(cudaFree(ds->host_stage));
+    for (cudaEvent_t ev : ds->aux_ev)
+        if (ev) keep(cudaEventDestroy(ev));
+    if (ds->aux) keep(cudaStreamDestroy(ds->aux));
     for (cudaEvent_t ev : ds->events) keep(cudaEventDestroy(ev));
     delete ds;
     return from_cuda(first);
@@ -694,6 +744,67 @@ nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_t B, int3
     if (st != NEST_OK) return st;
     return run_mix(ds, s_out, idx_out, p_lm, B, r, mu, lambda, 0, 0.f, 1.f, nullptr, p_knn_out,
                    p_m_out, s);
+}
+
+nest_status_t nest_knn_step_host(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                                 const int64_t* seg_off, const float* p_lm, float mu,
+                                 float lambda, float* s_out, int64_t* idx_out, float* p_m_out,
+                                 void* stream)
+{
+    if (!ds || !q || !p_lm || !s_out || !idx_out || !p_m_out) return NEST_ERR_INVALID_ARG;
+    if (B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R) return NEST_ERR_INVALID_ARG;
+    if (!(lambda >= 0.f && lambda <= 1.f)) return NEST_ERR_INVALID_ARG;
+    const size_t q_bytes = (size_t)B * ds->row_bytes;
+    const size_t so_bytes = seg_off ? (size_t)(B + 1) * 8 : 0;
+    const size_t v_bytes = (size_t)B * ds->vocab * 4;
+    const size_t s_bytes = (size_t)B * r * 4, i_bytes = (size_t)B * r * 8;
+    const size_t off_so = round256(q_bytes), off_p = off_so + round256(so_bytes);
+    const size_t off_s = off_p + round256(v_bytes), off_i = off_s + round256(s_bytes);
+    const size_t off_m = off_i + round256(i_bytes), total = off_m + round256(v_bytes);
+    nest_status_t st = ensure_host_stage(ds, total);
+    if (st == NEST_OK) st = ensure_aux(ds);
+    if (st != NEST_OK) return st;
+    unsigned char* d = ds->host_stage;
+    const int64_t* d_so = seg_off ? reinterpret_cast<const int64_t*>(d + off_so) : nullptr;
+    const float* d_p = reinterpret_cast<const float*>(d + off_p);
+    float* d_s = reinterpret_cast<float*>(d + off_s);
+    int64_t* d_i = reinterpret_cast<int64_t*>(d + off_i);
+    float* d_m = reinterpret_cast<float*>(d + off_m);
+    cudaStream_t s = as_stream(stream), x = ds->aux;
+    cudaEvent_t ev_start = ds->aux_ev[0], ev_lm = ds->aux_ev[1], ev_search = ds->aux_ev[2];
+    // the queries go in on `stream` ahead of the search; p_LM goes in on the
+    // side stream while the search runs, and s / idx come back on it while
+    // the mix runs
+    cudaError_t e = cudaEventRecord(ev_start, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(x, ev_start, 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d, q, q_bytes, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && seg_off)
+        e = cudaMemcpyAsync(d + off_so, seg_off, so_bytes, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d + off_p, p_lm, v_bytes, cudaMemcpyHostToDevice, x);
+    if (e == cudaSuccess) e = cudaEventRecord(ev_lm, x);
+    if (e != cudaSuccess) return from_cuda(e);
+    st = nest_knn_search(ds, d, B, r, d_so, d_s, d_i, stream);
+    if (st != NEST_OK) {
+        (void)cudaStreamSynchronize(x);
+        return st;
+    }
+    e = cudaEventRecord(ev_search, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(x, ev_search, 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(s_out, d_s, s_bytes, cudaMemcpyDeviceToHost, x);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(idx_out, d_i, i_bytes, cudaMemcpyDeviceToHost, x);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ev_lm, 0);
+    if (e != cudaSuccess) {
+        (void)cudaStreamSynchronize(x);
+        return from_cuda(e);
+    }
+    st = nest_knn_mix(ds, d_s, d_i, d_p, B, r, mu, lambda, nullptr, d_m, stream);
+    if (st == NEST_OK) e = cudaMemcpyAsync(p_m_out, d_m, v_bytes, cudaMemcpyDeviceToHost, s);
+    const cudaError_t es = cudaStreamSynchronize(s);
+    const cudaError_t ex = cudaStreamSynchronize(x);
+    if (st != NEST_OK) return st;
+    if (e == cudaSuccess) e = es;
+    if (e == cudaSuccess) e = ex;
+    return from_cuda(e);
 }
 
 nest_status_t nest_knn_search_masked(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,

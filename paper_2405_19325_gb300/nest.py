@@ -42,6 +42,7 @@ SIGNATURES = {
     "nest_knn_mix": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _P, _P, _P]),
     "nest_knn_mix_rrc": (ctypes.c_int, [_P, _P, _P, _P, _I32, _I32, _F, _F, _F, _P, _P, _P, _P]),
     "nest_knn_step": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _F, _F, _P, _P, _P, _P, _P]),
+    "nest_knn_step_host": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _F, _F, _P, _P, _P, _P]),
     "nest_device_status": (ctypes.c_int, [_P, _P]),
     "nest_timing_enable": (ctypes.c_int, [_P, _I32]),
     "nest_timing_read": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_double),
@@ -96,6 +97,16 @@ def _dtype_code(t: torch.Tensor) -> int:
 def _dev(t: torch.Tensor, name: str, dtype=None) -> int:
     if not isinstance(t, torch.Tensor) or not t.is_cuda:
         raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _host(t: torch.Tensor, name: str, dtype=None) -> int:
+    if not isinstance(t, torch.Tensor) or t.is_cuda:
+        raise TypeError(f"{name} must be a host tensor")
     if dtype is not None and t.dtype != dtype:
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_contiguous():
@@ -295,39 +306,32 @@ class Datastore:
     def step_host(self, q_host: torch.Tensor, r: int, p_lm_host: torch.Tensor, mu: float,
                   lam: float, seg_off_host: torch.Tensor | None = None, staging: dict | None = None,
                   stream=None) -> dict:
-        """One step from host (pinned) inputs to host outputs, copies on the stream.
+        """One step from host inputs to host outputs in one C call (nest_knn_step_host).
 
-        The query batch, p_LM and segment offsets go host -> device, the step
-        runs, and p_M, s and idx come back device -> host; the call returns
-        after the stream has finished.  ``staging`` caches device and pinned
-        buffers between calls.
+        The library copies the query batch, p_LM and the segment offsets to
+        device buffers of its own, runs the step on ``stream`` and copies p_M,
+        s and idx back before returning.  Page-locked host tensors let the
+        copies run asynchronously.  ``staging`` caches the page-locked output
+        tensors between calls (they are overwritten by the next call).
         """
-        st = staging if staging is not None else {}
-        s = stream if stream is not None else torch.cuda.current_stream()
-        dev = torch.device("cuda", torch.cuda.current_device())
         B = q_host.shape[0]
-        if "q" not in st:
-            st["q"] = torch.empty(q_host.shape, dtype=q_host.dtype, device=dev)
-            st["p_lm"] = torch.empty(p_lm_host.shape, dtype=torch.float32, device=dev)
-            if seg_off_host is not None:
-                st["seg_off"] = torch.empty(B + 1, dtype=torch.int64, device=dev)
-            st["host_p_m"] = torch.empty(B, self.vocab, dtype=torch.float32).pin_memory()
-            st["host_s"] = torch.empty(B, r, dtype=torch.float32).pin_memory()
-            st["host_idx"] = torch.empty(B, r, dtype=torch.int64).pin_memory()
-            st["out"] = {}
-        with torch.cuda.stream(s):
-            st["q"].copy_(q_host, non_blocking=True)
-            st["p_lm"].copy_(p_lm_host, non_blocking=True)
-            so = None
-            if seg_off_host is not None:
-                st["seg_off"].copy_(seg_off_host, non_blocking=True)
-                so = st["seg_off"]
-            o = self.step(st["q"], r, st["p_lm"], mu, lam, seg_off=so, out=st["out"], stream=s)
-            st["host_p_m"].copy_(o["p_m"], non_blocking=True)
-            st["host_s"].copy_(o["s"], non_blocking=True)
-            st["host_idx"].copy_(o["idx"], non_blocking=True)
-        s.synchronize()
-        return {"p_m": st["host_p_m"], "s": st["host_s"], "idx": st["host_idx"]}
+        if q_host.dtype != self.dtype or q_host.dim() != 2 or q_host.shape[1] != self.d:
+            raise ValueError("q must be B x d with the datastore's dtype")
+        if p_lm_host.dim() != 2 or p_lm_host.shape[0] != B or p_lm_host.shape[1] != self.vocab:
+            raise ValueError(f"p_lm must be {B} x {self.vocab}")
+        st = staging if staging is not None else {}
+        if st.get("shape") != (B, r):
+            st["shape"] = (B, r)
+            st["p_m"] = torch.empty(B, self.vocab, dtype=torch.float32).pin_memory()
+            st["s"] = torch.empty(B, r, dtype=torch.float32).pin_memory()
+            st["idx"] = torch.empty(B, r, dtype=torch.int64).pin_memory()
+        sp = _host(seg_off_host, "seg_off", torch.int64) if seg_off_host is not None else None
+        _check(self._lib.nest_knn_step_host(self._h, _host(q_host, "q"), B, r, sp,
+                                            _host(p_lm_host, "p_lm", torch.float32), float(mu),
+                                            float(lam), st["s"].data_ptr(), st["idx"].data_ptr(),
+                                            st["p_m"].data_ptr(), _stream(stream)),
+               "nest_knn_step_host")
+        return {"p_m": st["p_m"], "s": st["s"], "idx": st["idx"]}
 
     # ------------------------------------------------------------ status / timing
     def device_status(self, stream=None) -> int:

@@ -87,6 +87,13 @@ def test_search_and_mix_validation(lib):
     assert lib.nest_knn_mix_rrc(ds, s, i, p, 1, 1, 1.0, 0.3, 0.0, None, None, p, None) == 1
     assert lib.nest_knn_mix_rrc(ds, s, i, p, 1, 1, 1.0, 0.3, -1.0, None, None, p, None) == 1
     assert lib.nest_knn_step(ds, q, 1, 1, None, p, 1.0, 2.0, s, i, None, p, None) == 1
+    h = P(FAKE)  # host-pointer entry point: checks run before any device work
+    assert lib.nest_knn_step_host(None, h, 1, 1, None, h, 1.0, 0.5, h, h, h, None) == 1
+    assert lib.nest_knn_step_host(ds, None, 1, 1, None, h, 1.0, 0.5, h, h, h, None) == 1
+    assert lib.nest_knn_step_host(ds, h, 0, 1, None, h, 1.0, 0.5, h, h, h, None) == 1
+    assert lib.nest_knn_step_host(ds, h, 1, 4097, None, h, 1.0, 0.5, h, h, h, None) == 1
+    assert lib.nest_knn_step_host(ds, h, 1, 1, None, h, 1.0, 2.0, h, h, h, None) == 1
+    assert lib.nest_knn_step_host(ds, h, 1, 1, None, h, 1.0, 0.5, h, h, None, None) == 1
     assert lib.nest_knn_step(ds, q, 1, 1, None, p, 1.0, 0.5, None, i, None, p, None) == 1
 
 

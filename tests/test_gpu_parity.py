@@ -288,12 +288,35 @@ def test_timing_and_launch_count(nest):
 
 
 def test_step_host_matches_device_step(nest):
+    """nest_knn_step_host (host buffers in and out, one C call) gives the same
+    bytes as nest_knn_step on device copies: pinned and pageable inputs, two
+    batch sizes in a row (its device buffers grow), and a ragged batch."""
+    dev = torch.device("cuda")
     w = synth.WORKLOADS["tiny"]
     x = synth.make_inputs(w)
-    dev = torch.device("cuda")
     ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
-    host = ds.step_host(x.q.pin_memory(), w.r, x.p_lm.pin_memory(), w.mu, w.lam)
-    o = ds.step(x.q.to(dev), w.r, x.p_lm.to(dev), w.mu, w.lam)
+    staging = {}
+    for B, pin in ((w.B, True), (3, False), (w.B, True)):
+        q, p = x.q[:B].contiguous(), x.p_lm[:B].contiguous()
+        if pin:
+            q, p = q.pin_memory(), p.pin_memory()
+        host = ds.step_host(q, w.r, p, w.mu, w.lam, staging=staging)
+        o = ds.step(q.to(dev), w.r, p.to(dev), w.mu, w.lam)
+        torch.cuda.synchronize()
+        assert ds.device_status() == 0
+        assert torch.equal(host["p_m"], o["p_m"].cpu())
+        assert torch.equal(host["s"], o["s"].cpu())
+        assert torch.equal(host["idx"], o["idx"].cpu())
+    ds.close()
+
+    w = synth.WORKLOADS["ragged"]
+    x = synth.make_inputs(w, B=5)
+    ds = nest.Datastore(x.K.to(dev), x.V.to(dev), w.vocab)
+    host = ds.step_host(x.q.pin_memory(), w.r, x.p_lm.pin_memory(), w.mu, w.lam,
+                        seg_off_host=x.seg_off.pin_memory())
+    o = ds.step(x.q.to(dev), w.r, x.p_lm.to(dev), w.mu, w.lam, seg_off=x.seg_off.to(dev))
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
     assert torch.equal(host["p_m"], o["p_m"].cpu())
     assert torch.equal(host["idx"], o["idx"].cpu())
     ds.close()
