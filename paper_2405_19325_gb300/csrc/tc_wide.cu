@@ -31,17 +31,18 @@ constexpr int kMaxStagesW = 12;
 constexpr int kEpiThreads = 128;
 constexpr int kSelThreads = 1024;
 
-constexpr int kMaxEpiWarps = 8;
+constexpr int kMaxEpiWarps = 16;
 constexpr int kStageK = 4;  // admitted keys a lane stages per 32-column block
 
 template <int NM>
 struct WideShared {
     float qn[NM];      // ||q||^2 of the group's queries
     uint32_t thr[NM];  // a key is admitted iff the fp32 bits of its distance are <= thr
-    // Slots [x, y) of query column c's global list reserved by epilogue warp
-    // w and not yet written (used when WideArgs::resv > 0); x passes y once
-    // the block is used up.
-    int2 resv[kMaxEpiWarps][NM];
+    // Slots [x, y) of query column c's global list reserved by an epilogue
+    // warp and not yet written (used when WideArgs::resv > 0); x passes y
+    // once the block is used up.  Each warp has one entry per column it
+    // drains (NM / 2 or NM columns).
+    int2 resv[8 * NM];
     // Distance bits of the keys a lane admitted in one 32-column block, in
     // column order: [warp][k][lane].
     uint32_t stage[kMaxEpiWarps][kStageK][32];
@@ -199,13 +200,12 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
     }
 }
 
-// First reservations: lane i reserves a.resv slots in each column i + 32k of
-// the group for this warp (its atomics all in flight together).
-template <int NM>
-__device__ __forceinline__ void wide_reserve(int2* resv, int nqv, int lane, const WideArgs& a,
-                                             int q0)
+// First reservations: lane i reserves a.resv slots in each column
+// c_begin + i + 32k < c_end for this warp (its atomics all in flight together).
+__device__ __forceinline__ void wide_reserve(int2* resv, int c_begin, int c_end, int nqv, int lane,
+                                             const WideArgs& a, int q0)
 {
-    for (int c = lane; c < NM; c += 32) {
+    for (int c = c_begin + lane; c < c_end; c += 32) {
         int2 rv = make_int2(0, 0);
         if (a.resv > 0 && c < nqv) {
             rv.x = atomicAdd(&a.cnt[q0 + c], a.resv);
@@ -217,50 +217,67 @@ __device__ __forceinline__ void wide_reserve(int2* resv, int nqv, int lane, cons
 }
 
 // Pads what is left of this warp's blocks once the pass is done.
-template <int NM>
-__device__ __forceinline__ void wide_release(const int2* resv, int nqv, int lane, const WideArgs& a,
-                                             int q0)
+__device__ __forceinline__ void wide_release(const int2* resv, int c_begin, int c_end, int nqv,
+                                             int lane, const WideArgs& a, int q0)
 {
     if (a.resv <= 0) return;
     __syncwarp();
-    for (int c = lane; c < nqv && c < NM; c += 32) {
+    for (int c = c_begin + lane; c < nqv && c < c_end; c += 32) {
         const int2 rv = resv[c];
         if (rv.x < rv.y) wide_pad(a, q0 + c, rv.x, rv.y);
     }
 }
 
-// Drains one TMEM lane (this thread's key row) of an NM-column accumulator
-// at tbase, 32 columns per load with the next load in flight, and arrives
-// on `release` once the whole accumulator has been read.
-template <int NM>
-__device__ __forceinline__ void wide_drain_row(uint32_t tbase, uint64_t* release, int nqv, float kn,
-                                               bool valid, uint32_t key_idx, int lane,
-                                               const WideShared<NM>& sh, int2* resv,
+// Drains NCOL columns (queries c_base ..) of one TMEM lane (this thread's
+// key row) of an accumulator, starting at tbase, 32 columns per load, and
+// arrives on `release` once they have been read.  With PIPE the next load is
+// in flight while the current columns are tested (more registers); without
+// it the other warps of the SM sub-partition hide the load latency.
+template <int NM, int NCOL, bool PIPE>
+__device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint64_t* release,
+                                               int nqv, float kn, bool valid, uint32_t key_idx,
+                                               int lane, const WideShared<NM>& sh, int2* resv,
                                                uint32_t* stage, const WideArgs& a, int q0)
 {
-    static_assert(NM % 64 == 0 || NM == 32, "columns are drained in pairs of 32");
+    static_assert(NCOL % 64 == 0 || NCOL == 32, "columns are drained in pairs of 32");
+    if constexpr (!PIPE) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < NCOL; c0 += 32) {
+            uint32_t acc[32];
+            tmem_ld_32_async(tbase + (uint32_t)c0, acc);
+            tmem_wait_ld(acc);
+            if (c0 + 32 == NCOL) {
+                tc_fence_before();
+                mbar_arrive(release);
+            }
+            wide_columns<32, NM>(acc, c_base + c0, nqv, kn, valid, key_idx, lane, sh, resv, stage,
+                                 a, q0);
+        }
+        return;
+    }
     uint32_t a0[32], a1[32];
     tmem_ld_32_async(tbase, a0);
 #pragma unroll 1
-    for (int c0 = 0; c0 < NM; c0 += 64) {
+    for (int c0 = 0; c0 < NCOL; c0 += 64) {
         tmem_wait_ld(a0);
-        if (c0 + 32 < NM) {
+        if (c0 + 32 < NCOL) {
             tmem_ld_32_async(tbase + (uint32_t)(c0 + 32), a1);
         } else {
             tc_fence_before();
             mbar_arrive(release);
         }
-        wide_columns<32, NM>(a0, c0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a, q0);
-        if (c0 + 32 < NM) {
+        wide_columns<32, NM>(a0, c_base + c0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a,
+                             q0);
+        if (c0 + 32 < NCOL) {
             tmem_wait_ld(a1);
-            if (c0 + 64 < NM) {
+            if (c0 + 64 < NCOL) {
                 tmem_ld_32_async(tbase + (uint32_t)(c0 + 64), a0);
             } else {
                 tc_fence_before();
                 mbar_arrive(release);
             }
-            wide_columns<32, NM>(a1, c0 + 32, nqv, kn, valid, key_idx, lane, sh, resv, stage, a,
-                                    q0);
+            wide_columns<32, NM>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, lane, sh, resv,
+                                 stage, a, q0);
         }
     }
 }
@@ -418,9 +435,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (lane == 0) sh.qn[j] = s;
         }
         named_barrier(2, kEpiThreads);
-        int2* resv = sh.resv[warp - 2];
+        int2* resv = sh.resv + (warp - 2) * NM;
         uint32_t* stage = &sh.stage[warp - 2][0][0];
-        wide_reserve<NM>(resv, nqv, lane, a, q0);
+        wide_reserve(resv, 0, NM, nqv, lane, a, q0);
 
         const int row_in_tile = 32 * quarter + lane;
         const int64_t ks = a.key_stride;  // row i of the tensor map is key i * ks
@@ -443,11 +460,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 mbar_arrive(&sh.acc_empty[buf]);
                 wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a, q0);
             } else {
-                wide_drain_row<NM>(tbase, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane, sh,
-                                   resv, stage, a, q0);
+                wide_drain_row<NM, NM, true>(tbase, 0, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane,
+                                       sh, resv, stage, a, q0);
             }
         }
-        wide_release<NM>(resv, nqv, lane, a, q0);
+        wide_release(resv, 0, NM, nqv, lane, a, q0);
     }
 
     tc_fence_before();
@@ -468,9 +485,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // so one 64 KiB stage (32 KiB of keys, 32 KiB of queries) carries twice the
 // MMA work of a one-tile stage and the stage ring covers twice the latency.
 // The two 256-column fp32 accumulators fill TMEM, so a tile pair's epilogue
-// runs between its last MMA and the next pair's first; eight epilogue warps
-// (two per TMEM lane quarter, one per tile) keep that gap short.
-constexpr int kWide2Threads = 64 + 2 * kEpiThreads;
+// runs between its last MMA and the next pair's first; sixteen epilogue
+// warps (four per TMEM lane quarter: one per tile and half of the columns)
+// keep that gap short.
+constexpr int kWide2Epi = 4 * kEpiThreads;
+constexpr int kWide2Threads = 64 + kWide2Epi;
 
 __global__ void __launch_bounds__(kWide2Threads, 1)
     tc_wide2_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
@@ -506,7 +525,7 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             mbar_init(&sh.empty[s], 1);
         }
         mbar_init(&sh.acc_full[0], 1);
-        mbar_init(&sh.acc_empty[0], 2 * kEpiThreads);
+        mbar_init(&sh.acc_empty[0], kWide2Epi);
         mbar_init(&sh.drain, 1);
         sh.abort = 0;
         sh.issued = 0;
@@ -585,10 +604,12 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        const int e = tid - 64;  // 0 .. 255
+        const int e = tid - 64;  // 0 .. 511
+        const int ew = warp - 2;  // 0 .. 15
         const int quarter = warp & 3;
-        const int h = (warp - 2) >> 2;  // key tile of the pair this warp drains
-        for (int j = e; j < NM; j += 2 * kEpiThreads) {
+        const int h = (ew >> 2) & 1;            // key tile of the pair this warp drains
+        const int c_base = (ew >> 3) * (NM / 2);  // first of the NM / 2 columns it drains
+        for (int j = e; j < NM; j += kWide2Epi) {
             uint32_t thr = 0xFFFFFFFFu;
             if (a.s_sample != nullptr && j < nqv) {
                 const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
@@ -598,7 +619,7 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
         }
         const unsigned char* qb = static_cast<const unsigned char*>(a.q);
         const int chunks = a.d / 8;
-        for (int j = warp - 2; j < NM; j += 8) {
+        for (int j = ew; j < NM; j += kWide2Epi / 32) {
             float s = 0.f;
             if (j < nqv) {
                 const unsigned char* row = qb + (size_t)(q0 + j) * a.d * 2;
@@ -618,23 +639,25 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
             if (lane == 0) sh.qn[j] = s;
         }
-        named_barrier(2, 2 * kEpiThreads);
-        int2* resv = sh.resv[warp - 2];
-        uint32_t* stage = &sh.stage[warp - 2][0][0];
-        wide_reserve<NM>(resv, nqv, lane, a, q0);
+        named_barrier(2, kWide2Epi);
+        // this warp's reservation entries, indexed by the absolute column
+        int2* resv = sh.resv + ew * (NM / 2) - c_base;
+        uint32_t* stage = &sh.stage[ew][0][0];
+        wide_reserve(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
 
         const int64_t ks = a.key_stride;
-        const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM);
+        const uint32_t tbase =
+            tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM + c_base);
         for (int j = 0; j < npairs; ++j) {
             const int64_t row = lo + (int64_t)j * kPairKeys + h * kTileM + 32 * quarter + lane;
             const float kn = row < hi ? __ldg(a.knorm + row * ks) : 0.f;
             const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
             wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
             tc_fence_after();
-            wide_drain_row<NM>(tbase, &sh.acc_empty[0], nqv, kn, valid, (uint32_t)(row * ks), lane,
-                               sh, resv, stage, a, q0);
+            wide_drain_row<NM, NM / 2, false>(tbase, c_base, &sh.acc_empty[0], nqv, kn, valid,
+                                       (uint32_t)(row * ks), lane, sh, resv, stage, a, q0);
         }
-        wide_release<NM>(resv, nqv, lane, a, q0);
+        wide_release(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
     }
 
     tc_fence_before();
