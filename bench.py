@@ -287,13 +287,13 @@ def run_reference(args, w, world, rank):
 # capture summarised in profiles/tc_scan_decode_d4096_B4.md: 65,536-key case
 # scaled to the default 1,048,576 keys (reads x16, per-CTA writes unscaled).
 # Only valid for that kernel version on the default decode workload.
-DECODE_TC_SCAN_TRAFFIC = 537.27e6 * 16 + 3.05e6
+DECODE_TC_SCAN_TRAFFIC = 537.278464e6 * 16 + 3.055104e6
 
 # Same for the large-batch main pass, from profiles/tc_wide2_large_batch_B512.md:
 # the 262,144-key case scaled by 16 to the default 4,194,304 keys (key reads
 # and, with the sample size fixed at 65,536 keys, survivor writes both grow
 # with N).  Only valid for that kernel version on the default large batch.
-LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.339577e9 + 22.096384e6) * 16
+LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.359914e9 + 23.681280e6) * 16
 
 
 def dram_traffic(w, args, kernel):
