@@ -75,6 +75,7 @@ struct SearchPlan {
     int64_t sample_rows;
     bool single_pass;         // the sample is the whole datastore
     int64_t cap_s, cap_m;     // list capacities per query
+    int32_t resv;             // main pass: list slots an epilogue warp reserves at a time
     size_t off_cnt, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
 };
 
@@ -176,7 +177,21 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             sp->wpm.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
             sp->cap_s = sp->sample_rows;
             const int64_t expect = (ds->N * (int64_t)r + sp->sample_rows - 1) / sp->sample_rows;
-            sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect));
+            // Main-pass lists hold 8x the expected survivors plus what the
+            // epilogue warps' reservations can leave unwritten.  About a
+            // fraction r / sample_rows of the keys pass the sample's r-th
+            // distance, so a warp that drains `rows` key rows admits about
+            // rows * r / sample_rows keys per query; it reserves twice that
+            // plus 16 slots at a time (one atomic per block).  Each column
+            // has 4 reserving warps per CTA (8 with two key tiles per stage).
+            const int epi_warps = wp.mb == 2 ? 8 : 4;
+            const int64_t unit = (int64_t)kTcTileKeys * wp.mb;
+            const int64_t units = (ds->N + unit - 1) / unit;
+            const int64_t rows = (units + sp->wpm.parts - 1) / sp->wpm.parts * 32;
+            const int64_t per_warp = (rows * r + sp->sample_rows - 1) / sp->sample_rows;
+            sp->resv = (int32_t)std::min<int64_t>(2 * per_warp + 16, 1024);
+            const int64_t unwritten = (int64_t)sp->wpm.parts * epi_warps * sp->resv;
+            sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect)) + unwritten;
             sp->off_cnt = 0;  // 2 * B int32 counters
             sp->off_cand_s = (size_t)B;
             sp->off_s_s = sp->off_cand_s + (size_t)B * sp->cap_s;
@@ -339,26 +354,6 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
 
 // Large query batches: [sample pass, selection of the sample,] thresholded
 // pass over all keys, exact selection of the survivors.
-// List slots each epilogue warp of the main pass reserves per query at a
-// time.  About a fraction r / sample_rows of the keys pass the sample's r-th
-// distance, so a warp that drains `rows` key rows admits about
-// rows * r / sample_rows keys per query; it reserves twice that plus 16,
-// limited so that the first blocks of all warps leave room for twice the
-// expected survivors in the list.  Below 8 slots it is not worth it (0: one
-// atomic per admitting column).
-int32_t wide_reservation(const SearchPlan& sp, int64_t N, int32_t r)
-{
-    const int epi_warps = sp.wpm.mb == 2 ? 8 : 4;
-    const int64_t unit = (int64_t)kTcTileKeys * sp.wpm.mb;
-    const int64_t units = (N + unit - 1) / unit;
-    const int64_t rows = (units + sp.wpm.parts - 1) / sp.wpm.parts * 32;
-    const int64_t per_warp = (rows * r + sp.sample_rows - 1) / sp.sample_rows;
-    const int64_t expect = (N * r + sp.sample_rows - 1) / sp.sample_rows;
-    const int64_t room = (sp.cap_m - 2 * expect) / ((int64_t)sp.wpm.parts * epi_warps);
-    const int64_t R = std::min<int64_t>(2 * per_warp + 16, room);
-    return R >= 8 ? (int32_t)std::min<int64_t>(R, 1 << 20) : 0;
-}
-
 nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* q, int32_t B,
                           int32_t r, const uint32_t* key_mask, float* s_out, int64_t* idx_out,
                           uint64_t* scratch, bool timed, cudaStream_t stream)
@@ -440,7 +435,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     wa.N = ds->N;
     wa.parts = sp.wpm.parts;
     wa.key_stride = 1;
-    wa.resv = wide_reservation(sp, ds->N, r);
+    wa.resv = sp.resv;
     if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
     e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
     if (e != cudaSuccess) return from_cuda(e);

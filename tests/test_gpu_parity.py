@@ -359,6 +359,28 @@ def test_two_tile_wide_kernel_edges(nest, N, d, B, r):
     run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 900, "bf16", check_rows=rows)
 
 
+def test_wide_batch_keys_stored_cluster_by_cluster(nest):
+    """Keys stored cluster after cluster (as a datastore built document by
+    document would be): each query's main-pass survivors come from the one or
+    two key ranges that hold its cluster, so the epilogue warps there use up
+    their reserved list slots and go on one slot at a time.  bf16, d=256,
+    N=262,144 in 64 contiguous clusters, B=512, r=256."""
+    N, d, B, r, vocab = 262144, 256, 512, 256, 900
+    g = torch.Generator().manual_seed(31)
+    c = torch.randn(64, d, generator=g)
+    assign = torch.arange(N) // (N // 64)
+    K = (c[assign] + 0.3 * torch.randn(N, d, generator=g)).to(torch.bfloat16)
+    q = (c[torch.randint(0, 64, (B,), generator=g)]
+         + 0.3 * torch.randn(B, d, generator=g)).to(torch.bfloat16)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g) * 2, dim=1)
+    ds = nest.Datastore(K.cuda(), V.cuda(), vocab)
+    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.close()
+    rows = list(range(0, B, 37)) + [B - 1]
+    run_and_check(nest, K, V, q, p_lm, r, 1 / 16, 0.8, vocab, "bf16", check_rows=rows)
+
+
 def test_large_batch_shape_sampled_rows(nest):
     """Large-batch shape: bf16 d=4096, B=512, r=256, clustered keys (N reduced
     to 524,288); the oracle checks 12 query rows spread over the batch."""
