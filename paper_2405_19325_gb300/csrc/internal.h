@@ -157,6 +157,7 @@ struct GselectArgs {
     int32_t B;
     float* s_out;      // B x r
     int64_t* idx_out;  // B x r
+    int32_t stage_words;  // shared-memory words per CTA (set by launch_gselect)
 };
 
 bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* plan);

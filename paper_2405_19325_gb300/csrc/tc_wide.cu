@@ -674,38 +674,184 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
 }
 
 // ---------------------------------------------------------------- exact top-r of each global list
+// One CTA per query.  Three streaming passes over the query's list (eight
+// loads in flight per thread) replace a radix select in global memory:
+//   1. the number of real words (reserved slots never written hold
+//      kNoCandidate) and the least and greatest distance halves;
+//   2. a 2048-bin histogram of the 11 bits below the leading bits all real
+//      words share, which locates the bin b* holding the r-th smallest;
+//   3. every real word of a bin <= b* is copied to shared memory.
+// The bins order the words (same leading bits), so the copied words hold the
+// r smallest; the exact select and the sort then run in shared memory.  A
+// list with few real words is copied whole; if the bins up to b* hold more
+// words than shared memory takes, the radix select runs on the list in place.
+constexpr int kGselBins = 2048;
+constexpr int kGselUnroll = 8;
+
 struct GselShared {
     int cnt;
     uint64_t thr;
+    uint32_t hmin, hmax;
+    int nreal, take, bstar, upto;
+    int wsum[kSelThreads / 32];
+    uint32_t hist[kGselBins];
     SelectSmem<kSelThreads, 1> sel;
 };
 
-__global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectArgs a)
+// Copies the real words of list[0, n) that `keep` accepts into stage[]
+// (order not kept; the caller sorts).  Returns after a barrier.
+template <class Keep>
+__device__ __forceinline__ void gsel_copy(const uint64_t* list, int n, uint64_t* stage,
+                                          GselShared& sh, int tid, Keep keep)
 {
-    extern __shared__ __align__(16) uint64_t sort_buf[];  // next_pow2(r) words
-    __shared__ GselShared sh;
-    const int tid = threadIdx.x;
-    const int q = blockIdx.x;
-    uint64_t* list = a.cand + (int64_t)q * a.cap;
-    if (tid == 0) {
-        const int c = a.cnt[q];
-        sh.cnt = c < a.cap ? c : (int)a.cap;
-        sh.thr = kNoCandidate;
+    const int lane = tid & 31;
+    for (int base = tid; base < n; base += kGselUnroll * kSelThreads) {
+        uint64_t v[kGselUnroll];
+#pragma unroll
+        for (int u = 0; u < kGselUnroll; ++u) {
+            const int j = base + u * kSelThreads;
+            v[u] = j < n ? list[j] : kNoCandidate;
+        }
+#pragma unroll
+        for (int u = 0; u < kGselUnroll; ++u) {
+            const bool k = v[u] != kNoCandidate && keep(v[u]);
+            const uint32_t bal = __ballot_sync(~0u, k);
+            if (bal == 0) continue;
+            int at = 0;
+            if (lane == __ffs(bal) - 1) at = atomicAdd(&sh.take, __popc(bal));
+            at = __shfl_sync(~0u, at, __ffs(bal) - 1);
+            if (k) stage[at + __popc(bal & lanemask_lt())] = v[u];
+        }
     }
     __syncthreads();
-    // keeps the r smallest at the front of the list, in place
-    select_smallest<kSelThreads, 1>(list, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
-                                    [] { __syncthreads(); });
-    const int n = sh.cnt;
-    int P2 = 1;
-    while (P2 < (n > 0 ? n : 1)) P2 <<= 1;
-    for (int j = tid; j < P2; j += kSelThreads) sort_buf[j] = j < n ? list[j] : kNoCandidate;
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectArgs a)
+{
+    extern __shared__ __align__(16) uint64_t stage[];  // a.stage_words words
+    __shared__ GselShared sh;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int q = blockIdx.x;
+    uint64_t* list = a.cand + (int64_t)q * a.cap;
+    const int c = a.cnt[q];
+    const int n = c < a.cap ? c : (int)a.cap;
+    if (tid == 0) {
+        sh.hmin = ~0u;
+        sh.hmax = 0;
+        sh.nreal = 0;
+        sh.take = 0;
+        sh.thr = kNoCandidate;
+    }
+    for (int i = tid; i < kGselBins; i += kSelThreads) sh.hist[i] = 0;
     __syncthreads();
-    bitonic_sort<kSelThreads>(sort_buf, P2, tid, [] { __syncthreads(); });
+
+    // 1. real words and the range of their distance halves
+    {
+        uint32_t lo = ~0u, hi = 0, cnt = 0;
+        for (int base = tid; base < n; base += kGselUnroll * kSelThreads) {
+            uint64_t v[kGselUnroll];
+#pragma unroll
+            for (int u = 0; u < kGselUnroll; ++u) {
+                const int j = base + u * kSelThreads;
+                v[u] = j < n ? list[j] : kNoCandidate;
+            }
+#pragma unroll
+            for (int u = 0; u < kGselUnroll; ++u) {
+                if (v[u] == kNoCandidate) continue;
+                const uint32_t h = (uint32_t)(v[u] >> 32);
+                lo = h < lo ? h : lo;
+                hi = h > hi ? h : hi;
+                ++cnt;
+            }
+        }
+        lo = __reduce_min_sync(~0u, lo);
+        hi = __reduce_max_sync(~0u, hi);
+        cnt = __reduce_add_sync(~0u, cnt);
+        if (lane == 0) {
+            atomicMin(&sh.hmin, lo);
+            atomicMax(&sh.hmax, hi);
+            atomicAdd(&sh.nreal, (int)cnt);
+        }
+    }
+    __syncthreads();
+    const int nreal = sh.nreal;
+    int m = -1;  // words staged in shared memory; -1: select in place
+    if (nreal <= a.stage_words && nreal <= 4 * a.r) {
+        gsel_copy(list, n, stage, sh, tid, [](uint64_t) { return true; });
+        m = sh.take;
+    } else {
+        const uint32_t x = sh.hmin ^ sh.hmax;
+        const int L = x ? __clz(x) : 32;  // leading bits all real words share
+        const int shift = 53 - L;          // the 11 bits below them
+        // 2. histogram
+        for (int base = tid; base < n; base += kGselUnroll * kSelThreads) {
+            uint64_t v[kGselUnroll];
+#pragma unroll
+            for (int u = 0; u < kGselUnroll; ++u) {
+                const int j = base + u * kSelThreads;
+                v[u] = j < n ? list[j] : kNoCandidate;
+            }
+#pragma unroll
+            for (int u = 0; u < kGselUnroll; ++u)
+                if (v[u] != kNoCandidate)
+                    atomicAdd(&sh.hist[(uint32_t)(v[u] >> shift) & (kGselBins - 1)], 1u);
+        }
+        __syncthreads();
+        // the bin holding the r-th smallest (thread t: bins 2t, 2t + 1)
+        const uint32_t h0 = sh.hist[2 * tid], h1 = sh.hist[2 * tid + 1];
+        uint32_t incl = h0 + h1;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(~0u, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) sh.wsum[warp] = (int)incl;
+        __syncthreads();
+        uint32_t carry = 0;
+        for (int w = 0; w < warp; ++w) carry += (uint32_t)sh.wsum[w];
+        const uint32_t excl = carry + incl - (h0 + h1);
+        const uint32_t r = (uint32_t)a.r;
+        if (excl < r && r <= excl + h0 + h1) {
+            const bool first = excl + h0 >= r;
+            sh.bstar = first ? 2 * tid : 2 * tid + 1;
+            sh.upto = (int)(first ? excl + h0 : excl + h0 + h1);
+        }
+        __syncthreads();
+        if (sh.upto <= a.stage_words) {
+            // 3. the real words of bins <= b*
+            const uint32_t bstar = (uint32_t)sh.bstar;
+            gsel_copy(list, n, stage, sh, tid, [shift, bstar](uint64_t e) {
+                return ((uint32_t)(e >> shift) & (kGselBins - 1)) <= bstar;
+            });
+            m = sh.take;
+        }
+    }
+
+    int nsel;
+    if (m >= 0) {
+        if (tid == 0) sh.cnt = m;
+        __syncthreads();
+        select_smallest<kSelThreads, 1>(stage, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
+                                        [] { __syncthreads(); });
+        nsel = sh.cnt;
+    } else {
+        // keeps the r smallest at the front of the list, in place
+        if (tid == 0) sh.cnt = n;
+        __syncthreads();
+        select_smallest<kSelThreads, 1>(list, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
+                                        [] { __syncthreads(); });
+        nsel = sh.cnt;
+        for (int j = tid; j < nsel; j += kSelThreads) stage[j] = list[j];
+    }
+    int P2 = 1;
+    while (P2 < (nsel > 0 ? nsel : 1)) P2 <<= 1;
+    for (int j = nsel + tid; j < P2; j += kSelThreads) stage[j] = kNoCandidate;
+    __syncthreads();
+    bitonic_sort<kSelThreads>(stage, P2, tid, [] { __syncthreads(); });
     float* so = a.s_out + (int64_t)q * a.r;
     int64_t* io = a.idx_out + (int64_t)q * a.r;
     for (int j = tid; j < a.r; j += kSelThreads) {
-        const uint64_t e = j < n ? sort_buf[j] : kNoCandidate;
+        const uint64_t e = j < nsel ? stage[j] : kNoCandidate;
         if (e != kNoCandidate) {  // reserved slots never written hold kNoCandidate
             so[j] = -__uint_as_float((uint32_t)(e >> 32));
             io[j] = (int64_t)(uint32_t)e;
@@ -796,11 +942,13 @@ cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUte
     }
 }
 
-cudaError_t launch_gselect(const GselectArgs& a, cudaStream_t stream)
+cudaError_t launch_gselect(const GselectArgs& in, cudaStream_t stream)
 {
+    GselectArgs a = in;
     int P2 = 1;
     while (P2 < a.r) P2 <<= 1;
-    const size_t smem = (size_t)P2 * sizeof(uint64_t);
+    a.stage_words = P2 > 16384 ? P2 : 16384;  // at least next_pow2(r): the sort runs there
+    const size_t smem = (size_t)a.stage_words * sizeof(uint64_t);
     cudaError_t e = cudaFuncSetAttribute(gselect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
