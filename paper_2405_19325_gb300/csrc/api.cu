@@ -76,7 +76,7 @@ struct SearchPlan {
     bool single_pass;         // the sample is the whole datastore
     int64_t cap_s, cap_m;     // list capacities per query
     int32_t resv;             // main pass: list slots an epilogue warp reserves at a time
-    size_t off_cnt, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
+    size_t off_cnt, off_qn, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
 };
 
 // Parts per query group.  Time ~ waves * (work per part + fixed cost per part),
@@ -193,7 +193,8 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             const int64_t unwritten = (int64_t)sp->wpm.parts * epi_warps * sp->resv;
             sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect)) + unwritten;
             sp->off_cnt = 0;  // 2 * B int32 counters
-            sp->off_cand_s = (size_t)B;
+            sp->off_qn = (size_t)B;  // B floats: ||q||^2
+            sp->off_cand_s = sp->off_qn + ((size_t)B + 1) / 2;
             sp->off_s_s = sp->off_cand_s + (size_t)B * sp->cap_s;
             sp->off_i_s = sp->off_s_s + ((size_t)B * r + 1) / 2;
             sp->off_cand_m = sp->off_i_s + (size_t)B * r;
@@ -368,6 +369,8 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     WideArgs wa{};
     wa.knorm = ds->knorm;
     wa.q = q;
+    float* qn = reinterpret_cast<float*>(scratch + sp.off_qn);
+    wa.qn = qn;
     wa.key_mask = key_mask;
     wa.status = ds->status;
     wa.r = r;
@@ -376,6 +379,9 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     wa.groups = sp.wpm.groups;
     wa.stages = sp.wpm.stages;
     wa.kchunks = (ds->d + 63) / 64;
+    e = launch_wide_qnorm(q, B, ds->d, qn, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
 
     GselectArgs ga{};
     ga.r = r;

@@ -128,6 +128,7 @@ struct WidePlan {
 struct WideArgs {
     const float* knorm;
     const void* q;
+    const float* qn;  // B: ||q||^2 (launch_wide_qnorm)
     const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     int* status;
     const float* s_sample;  // B x r sample neighbours (threshold = s[r-1]); null: admit all
@@ -161,6 +162,8 @@ struct GselectArgs {
 };
 
 bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* plan);
+// ||q||^2 of B bf16 rows of d elements into qn (fp32, one warp per row).
+cudaError_t launch_wide_qnorm(const void* q, int32_t B, int32_t d, float* qn, cudaStream_t stream);
 cudaError_t launch_tc_wide(const WidePlan& plan, const CUtensorMap& keys,
                            const CUtensorMap& queries, const WideArgs& args, cudaStream_t stream);
 cudaError_t launch_gselect(const GselectArgs& args, cudaStream_t stream);

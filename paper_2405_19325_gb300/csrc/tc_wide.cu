@@ -87,7 +87,9 @@ __device__ __forceinline__ void wide_pad(const WideArgs& a, int64_t col, int fro
 // row: D = ||q||^2 + ||k||^2 - 2 q.k, clamped at 0, admitted at or below the
 // query's threshold.  The admission test is branch-free over the W columns.
 //
-// Appending, when some lane admits a key:
+// On the pass that admits every key (no thresholds), word positions are the
+// tensor-map rows, so no slots are taken.  Appending, when some lane admits a
+// key on a thresholded pass:
 //  * with reservations (a.resv > 0) and at most kStageK admitted keys per
 //    lane, a branch-free pass stages each lane's admitted distances in
 //    shared memory, then each lane takes a slot per key from this warp's
@@ -99,10 +101,30 @@ __device__ __forceinline__ void wide_pad(const WideArgs& a, int64_t col, int fro
 //    its word.
 template <int W, int NM>
 __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, int nqv, float kn,
-                                             bool valid, uint32_t key_idx, int lane,
+                                             bool valid, uint32_t key_idx, int64_t pos, int lane,
                                              const WideShared<NM>& sh, int2* resv,
                                              uint32_t* stage, const WideArgs& a, int q0)
 {
+    if (a.s_sample == nullptr) {
+        // every key is admitted: the word of tensor-map row `pos` goes to
+        // position `pos` of each list (masked keys leave a padding word)
+        if (pos < 0) return;
+#pragma unroll
+        for (int v = 0; v < W / 4; ++v) {
+            const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
+            const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int col = c0 + 4 * v + k;
+                float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
+                dist = (dist <= 0.f) ? 0.f : dist;
+                if (col < nqv)
+                    a.cand[(int64_t)(q0 + col) * a.cap + pos] =
+                        valid ? (((uint64_t)__float_as_uint(dist) << 32) | key_idx) : kNoCandidate;
+            }
+        }
+        return;
+    }
     uint32_t m = 0;
 #pragma unroll
     for (int v = 0; v < W / 4; ++v) {
@@ -236,7 +258,8 @@ __device__ __forceinline__ void wide_release(const int2* resv, int c_begin, int 
 template <int NM, int NCOL, bool PIPE>
 __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint64_t* release,
                                                int nqv, float kn, bool valid, uint32_t key_idx,
-                                               int lane, const WideShared<NM>& sh, int2* resv,
+                                               int64_t pos, int lane, const WideShared<NM>& sh,
+                                               int2* resv,
                                                uint32_t* stage, const WideArgs& a, int q0)
 {
     static_assert(NCOL % 64 == 0 || NCOL == 32, "columns are drained in pairs of 32");
@@ -250,7 +273,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
                 tc_fence_before();
                 mbar_arrive(release);
             }
-            wide_columns<32, NM>(acc, c_base + c0, nqv, kn, valid, key_idx, lane, sh, resv, stage,
+            wide_columns<32, NM>(acc, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage,
                                  a, q0);
         }
         return;
@@ -266,7 +289,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
             tc_fence_before();
             mbar_arrive(release);
         }
-        wide_columns<32, NM>(a0, c_base + c0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a,
+        wide_columns<32, NM>(a0, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage, a,
                              q0);
         if (c0 + 32 < NCOL) {
             tmem_wait_ld(a1);
@@ -276,7 +299,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
                 tc_fence_before();
                 mbar_arrive(release);
             }
-            wide_columns<32, NM>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, lane, sh, resv,
+            wide_columns<32, NM>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, pos, lane, sh, resv,
                                  stage, a, q0);
         }
     }
@@ -410,30 +433,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
             }
             sh.thr[j] = thr;
+            // the pass that admits every key fills whole lists (positions = rows)
+            if (a.s_sample == nullptr && part == 0 && j < nqv) a.cnt[q0 + j] = (int32_t)a.N;
         }
-        // ||q||^2 of the group's queries (warp w: queries w, w + 4, ...), bf16 values
-        const unsigned char* qb = static_cast<const unsigned char*>(a.q);
-        const int chunks = a.d / 8;  // 16-byte chunks of a row (d * 2 is a multiple of 16)
-        for (int j = warp - 2; j < NM; j += 4) {
-            float s = 0.f;
-            if (j < nqv) {
-                const unsigned char* row = qb + (size_t)(q0 + j) * a.d * 2;
-                for (int c = lane; c < chunks; c += 32) {
-                    const uint4 v = ld_global_nc_v4(row + (size_t)c * 16);
-                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float lo = __uint_as_float(w[i] << 16);
-                        const float hi = __uint_as_float(w[i] & 0xffff0000u);
-                        s = fmaf(lo, lo, s);
-                        s = fmaf(hi, hi, s);
-                    }
-                }
-            }
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
-            if (lane == 0) sh.qn[j] = s;
-        }
+        // ||q||^2 of the group's queries, computed once per search
+        for (int j = e; j < NM; j += kEpiThreads) sh.qn[j] = j < nqv ? a.qn[q0 + j] : 0.f;
         named_barrier(2, kEpiThreads);
         int2* resv = sh.resv + (warp - 2) * NM;
         uint32_t* stage = &sh.stage[warp - 2][0][0];
@@ -449,6 +453,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const float kn = kn_next;
             kn_next = (row + kTileM < hi) ? __ldg(a.knorm + (row + kTileM) * ks) : 0.f;
             const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
+            const int64_t pos = row < hi ? row : -1;
             wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
             tc_fence_after();
             const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);
@@ -458,9 +463,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tmem_ld_16(tbase, acc);
                 tc_fence_before();
                 mbar_arrive(&sh.acc_empty[buf]);
-                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, lane, sh, resv, stage, a, q0);
+                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage, a, q0);
             } else {
-                wide_drain_row<NM, NM, true>(tbase, 0, &sh.acc_empty[buf], nqv, kn, valid, key_idx, lane,
+                wide_drain_row<NM, NM, true>(tbase, 0, &sh.acc_empty[buf], nqv, kn, valid, key_idx, pos, lane,
                                        sh, resv, stage, a, q0);
             }
         }
@@ -616,29 +621,10 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
                 if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
             }
             sh.thr[j] = thr;
+            // the pass that admits every key fills whole lists (positions = rows)
+            if (a.s_sample == nullptr && part == 0 && j < nqv) a.cnt[q0 + j] = (int32_t)a.N;
         }
-        const unsigned char* qb = static_cast<const unsigned char*>(a.q);
-        const int chunks = a.d / 8;
-        for (int j = ew; j < NM; j += kWide2Epi / 32) {
-            float s = 0.f;
-            if (j < nqv) {
-                const unsigned char* row = qb + (size_t)(q0 + j) * a.d * 2;
-                for (int c = lane; c < chunks; c += 32) {
-                    const uint4 v = ld_global_nc_v4(row + (size_t)c * 16);
-                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float lo_ = __uint_as_float(w[i] << 16);
-                        const float hi_ = __uint_as_float(w[i] & 0xffff0000u);
-                        s = fmaf(lo_, lo_, s);
-                        s = fmaf(hi_, hi_, s);
-                    }
-                }
-            }
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
-            if (lane == 0) sh.qn[j] = s;
-        }
+        for (int j = e; j < NM; j += kWide2Epi) sh.qn[j] = j < nqv ? a.qn[q0 + j] : 0.f;
         named_barrier(2, kWide2Epi);
         // this warp's reservation entries, indexed by the absolute column
         int2* resv = sh.resv + ew * (NM / 2) - c_base;
@@ -652,10 +638,11 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             const int64_t row = lo + (int64_t)j * kPairKeys + h * kTileM + 32 * quarter + lane;
             const float kn = row < hi ? __ldg(a.knorm + row * ks) : 0.f;
             const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
+            const int64_t pos = row < hi ? row : -1;
             wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
             tc_fence_after();
             wide_drain_row<NM, NM / 2, false>(tbase, c_base, &sh.acc_empty[0], nqv, kn, valid,
-                                       (uint32_t)(row * ks), lane, sh, resv, stage, a, q0);
+                                       (uint32_t)(row * ks), pos, lane, sh, resv, stage, a, q0);
         }
         wide_release(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
     }
@@ -671,6 +658,35 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
         for (int s = max(0, issued - a.stages); s < issued; ++s)
             (void)mbar_wait_bounded(&sh.full[s % a.stages], (uint32_t)(s / a.stages) & 1u);
     }
+}
+
+// ---------------------------------------------------------------- query norms
+// ||q||^2 of each bf16 query row, one warp per row: lane l sums the squares
+// of 16-byte chunks l, l + 32, ... in order, then the warp adds the lanes'
+// sums by a butterfly.  Both passes of a search read the same values.
+__global__ void __launch_bounds__(256) wide_qnorm_kernel(const unsigned char* q, int32_t B,
+                                                         int32_t d, float* qn)
+{
+    const int lane = threadIdx.x & 31;
+    const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (j >= B) return;
+    const unsigned char* row = q + (size_t)j * d * 2;
+    const int chunks = d / 8;  // 16-byte chunks of a row (d * 2 is a multiple of 16)
+    float s = 0.f;
+    for (int c = lane; c < chunks; c += 32) {
+        const uint4 v = ld_global_nc_v4(row + (size_t)c * 16);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float lo = __uint_as_float(w[i] << 16);
+            const float hi = __uint_as_float(w[i] & 0xffff0000u);
+            s = fmaf(lo, lo, s);
+            s = fmaf(hi, hi, s);
+        }
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
+    if (lane == 0) qn[j] = s;
 }
 
 // ---------------------------------------------------------------- exact top-r of each global list
@@ -940,6 +956,13 @@ cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUte
     case 256: return wide_launch_nm<256>(p, tmK, tmQ, a, stream);
     default: return cudaErrorInvalidValue;
     }
+}
+
+cudaError_t launch_wide_qnorm(const void* q, int32_t B, int32_t d, float* qn, cudaStream_t stream)
+{
+    wide_qnorm_kernel<<<(B + 7) / 8, 256, 0, stream>>>(static_cast<const unsigned char*>(q), B, d,
+                                                       qn);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_gselect(const GselectArgs& in, cudaStream_t stream)
