@@ -37,7 +37,8 @@ constexpr int kStageK = 4;  // admitted keys a lane stages per 32-column block
 template <int NM>
 struct WideShared {
     float qn[NM];      // ||q||^2 of the group's queries
-    uint32_t thr[NM];  // a key is admitted iff the fp32 bits of its distance are <= thr
+    uint32_t thr[NM];  // a key is admitted iff the fp32 bits of its distance, as signed
+                       // integers, are <= thr (0xFFFFFFFF = -1 for padding columns)
     // Slots [x, y) of query column c's global list reserved by an epilogue
     // warp and not yet written (used when WideArgs::resv > 0); x passes y
     // once the block is used up.  Each warp has one entry per column it
@@ -125,52 +126,50 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
         }
         return;
     }
+    // Admission: the fp32 bits of D compared as signed integers with the
+    // query's threshold (thr[] >= 0; -1 for padding columns).  A negative D
+    // (rounding) has the sign bit set and is admitted, as the clamp to 0
+    // would; only stored words are clamped.  With reservations, each lane
+    // also stages its admitted distances in the same pass (predicated
+    // stores, no branch); slot kStageK and beyond are never written.
+    const bool staging = a.resv > 0;
+    uint32_t* st = stage + lane;
     uint32_t m = 0;
+    int n = 0;
 #pragma unroll
     for (int v = 0; v < W / 4; ++v) {
         const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
-        const uint4 tv = *reinterpret_cast<const uint4*>(sh.thr + c0 + 4 * v);
+        const int4 tv = *reinterpret_cast<const int4*>(sh.thr + c0 + 4 * v);
         const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
-        const uint32_t ta[4] = {tv.x, tv.y, tv.z, tv.w};
+        const int ta[4] = {tv.x, tv.y, tv.z, tv.w};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
-            dist = (dist <= 0.f) ? 0.f : dist;
-            m |= (__float_as_uint(dist) <= ta[k] ? 1u : 0u) << (4 * v + k);
-        }
-    }
-    // padding columns (no query) and rows past the range never append
-    const int ncol = nqv - c0;
-    const uint32_t colmask = ncol >= 32 ? ~0u : (ncol <= 0 ? 0u : (1u << ncol) - 1u);
-    m = valid ? (m & colmask) : 0u;
-    const uint32_t any = __reduce_or_sync(~0u, m);
-    if (any == 0) return;
-    if (a.resv > 0 && __all_sync(~0u, __popc(m) <= kStageK)) {
-        uint32_t* st = stage + lane;
-        int n = 0;
-#pragma unroll
-        for (int v = 0; v < W / 4; ++v) {
-            const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
-            const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
-                dist = (dist <= 0.f) ? 0.f : dist;
-                const int b = (m >> (4 * v + k)) & 1u;
-                st_shared_u32_if(b != 0, st + n * 32, __float_as_uint(dist));
-                n += b;
+            const float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
+            const bool b = valid && __float_as_int(dist) <= ta[k];
+            m |= (b ? 1u : 0u) << (4 * v + k);
+            if (staging) {
+                st_shared_u32_if(b && n < kStageK, st + n * 32, __float_as_uint(dist));
+                n += b ? 1 : 0;
             }
         }
+    }
+    const uint32_t any = __reduce_or_sync(~0u, m);
+    if (any == 0) return;
+    if (staging && __all_sync(~0u, n <= kStageK)) {
+        // each lane takes one slot per staged key from this warp's block for
+        // the column (a shared-memory atomic), or one fresh slot of the list
+        // once the block is used up
         __syncwarp();
         uint32_t mm = m;
         for (int j = 0; j < n; ++j) {
             const int col = c0 + __ffs(mm) - 1;
             mm &= mm - 1;
-            const uint32_t dbits = st[j * 32];
-            int pos = atomicAdd(&resv[col].x, 1);
-            if (pos >= resv[col].y) pos = atomicAdd(&a.cnt[q0 + col], 1);
-            if (pos < a.cap)
-                a.cand[(int64_t)(q0 + col) * a.cap + pos] = ((uint64_t)dbits << 32) | key_idx;
+            uint32_t dbits = st[j * 32];
+            dbits = (int)dbits < 0 ? 0u : dbits;  // D <= 0 is stored as 0
+            int slot = atomicAdd(&resv[col].x, 1);
+            if (slot >= resv[col].y) slot = atomicAdd(&a.cnt[q0 + col], 1);
+            if (slot < a.cap)
+                a.cand[(int64_t)(q0 + col) * a.cap + slot] = ((uint64_t)dbits << 32) | key_idx;
             else
                 record_status(a.status, NEST_ERR_OVERFLOW);
         }
@@ -427,10 +426,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // distance of the sample (an upper bound of the true r-th distance),
         // or every key on the sampling pass itself (no s_sample).
         for (int j = e; j < NM; j += kEpiThreads) {
+            // padding columns: -1 (never admitted); no sample threshold: every key
             uint32_t thr = 0xFFFFFFFFu;
-            if (a.s_sample != nullptr && j < nqv) {
-                const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
-                if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+            if (j < nqv) {
+                thr = 0x7FFFFFFFu;
+                if (a.s_sample != nullptr) {
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+                }
             }
             sh.thr[j] = thr;
             // the pass that admits every key fills whole lists (positions = rows)
@@ -615,10 +618,14 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
         const int h = (ew >> 2) & 1;            // key tile of the pair this warp drains
         const int c_base = (ew >> 3) * (NM / 2);  // first of the NM / 2 columns it drains
         for (int j = e; j < NM; j += kWide2Epi) {
+            // padding columns: -1 (never admitted); no sample threshold: every key
             uint32_t thr = 0xFFFFFFFFu;
-            if (a.s_sample != nullptr && j < nqv) {
-                const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
-                if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+            if (j < nqv) {
+                thr = 0x7FFFFFFFu;
+                if (a.s_sample != nullptr) {
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+                }
             }
             sh.thr[j] = thr;
             // the pass that admits every key fills whole lists (positions = rows)
