@@ -2,18 +2,24 @@
 // r nearest keys of each query, s = -||q - k||^2), where per-query candidate
 // lists no longer fit in one CTA's shared memory.
 //
-//   1. A sampling pre-pass: the same kernel over a tensor map that reads
-//      every stride-th key, admitting every sampled key, and gselect_kernel
-//      on those lists give each query the r-th distance among the sample.
-//      It is an upper bound of the query's true r-th distance, so every key
-//      at or below it is a safe candidate (admission threshold).
-//   2. tc_wide_kernel streams every key tile once per group of up to 256
-//      queries: tcgen05.mma with M = 128 keys, N = up to 256 queries,
-//      K = 16, two TMEM accumulators of N columns; the epilogue warps form
-//      ||q||^2 + ||k||^2 - 2 q.k and append the keys under each query's
-//      threshold to that query's global list (one atomic per warp and query).
-//   3. gselect_kernel takes the exact r smallest of each list (radix select
-//      in place in global memory), sorts them and writes s and idx.
+//   0. wide_qnorm_kernel computes ||q||^2 of every query once.
+//   1. A sampling pre-pass: the scan kernel over a tensor map that reads
+//      every stride-th key, admitting every sampled key (each list holds the
+//      sample in row order), and gselect_kernel on those lists give each
+//      query the r-th distance among the sample.  It is an upper bound of the
+//      query's true r-th distance, so every key at or below it is a safe
+//      candidate (admission threshold).
+//   2. The main pass streams every key tile once per group of up to 256
+//      queries with tcgen05.mma (M = 128 keys, N = up to 256 queries,
+//      K = 16): tc_wide_kernel keeps one key tile per stage and two TMEM
+//      accumulators of N columns; tc_wide2_kernel (groups of 256) keeps two
+//      key tiles per stage, one accumulator each.  The epilogue warps form
+//      ||q||^2 + ||k||^2 - 2 q.k, admit the keys under each query's threshold
+//      and append them to that query's global list through per-warp slot
+//      reservations.
+//   3. gselect_kernel takes the exact r smallest of each list (three
+//      streaming passes, then a select in shared memory), sorts them and
+//      writes s and idx.
 #include <cmath>
 #include <cuda.h>
 
