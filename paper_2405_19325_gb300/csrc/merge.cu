@@ -2,9 +2,8 @@
 // neighbours (the selection of pi, Sec. 2.2 / Algorithm 1's search step).
 //
 // A CTA copies the real entries of up to per_cta lists of one query into
-// shared memory (list lengths come with the lists, so the copy is one fully
-// parallel pass), keeps the r smallest words with the same radix select the
-// scan uses, and either writes them as one list for the next level or, on
+// shared memory (one warp per list, at offsets from the lists' lengths),
+// keeps the r smallest words with the same radix select the scan uses, and either writes them as one list for the next level or, on
 // the last level, sorts them (bitonic) and writes s = -distance and the key
 // index, nearest first, ties by smaller index, padding with (-inf, -1).
 #include <cmath>
