@@ -4,6 +4,8 @@
 #include <cstdlib>
 #include <cstring>
 #include <new>
+#include <map>
+#include <mutex>
 #include <vector>
 
 #include <cudaTypedefs.h>
@@ -277,7 +279,31 @@ nest_status_t record_event(nest_datastore* ds, cudaStream_t stream)
     return from_cuda(cudaEventRecord(ds->events[ds->events_used++], stream));
 }
 
-// Device pointers only: plain host memory would fault on GPUs that cannot reach it.
+}  // namespace
+
+cudaError_t nest::raise_smem_limit(const void* kernel, size_t smem)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    static std::mutex mu;
+    static std::map<std::pair<const void*, int>, size_t> limit;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        const auto it = limit.find({kernel, dev});
+        if (it != limit.end() && it->second >= smem) return cudaSuccess;
+    }
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) {
+        std::lock_guard<std::mutex> lock(mu);
+        size_t& v = limit[{kernel, dev}];
+        v = v > smem ? v : smem;
+    }
+    return e;
+}
+
+namespace {
+
 // Device buffers of nest_knn_step_host, grown on demand (never shrunk).
 nest_status_t ensure_host_stage(nest_datastore* ds, size_t bytes)
 {
@@ -320,6 +346,7 @@ nest_status_t ensure_aux(nest_datastore* ds)
     return NEST_OK;
 }
 
+// Device pointers only: plain host memory would fault on GPUs that cannot reach it.
 bool is_device_pointer(const void* p)
 {
     cudaPointerAttributes at;

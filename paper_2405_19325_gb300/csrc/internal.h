@@ -10,6 +10,11 @@
 
 namespace nest {
 
+// Raises a kernel's dynamic shared-memory limit on the current device when a
+// launch needs more than the largest size set for it so far (one driver
+// call per kernel and increase, not per launch).
+cudaError_t raise_smem_limit(const void* kernel, size_t smem);
+
 // A candidate neighbour is one 64-bit word: the fp32 bits of its squared
 // distance (non-negative, so the bits order like the values) above its
 // 32-bit key index.  Ordering the words orders neighbours nearest first

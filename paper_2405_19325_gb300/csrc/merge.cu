@@ -161,13 +161,11 @@ cudaError_t launch_merge(const MergeArgs& a, bool last, cudaStream_t stream)
     const dim3 grid(groups, a.B);
     cudaError_t e;
     if (last) {
-        e = cudaFuncSetAttribute(merge_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
+        e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel<true>), (int)smem);
         if (e != cudaSuccess) return e;
         merge_kernel<true><<<grid, kMergeThreads, smem, stream>>>(a);
     } else {
-        e = cudaFuncSetAttribute(merge_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
+        e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel<false>), (int)smem);
         if (e != cudaSuccess) return e;
         merge_kernel<false><<<grid, kMergeThreads, smem, stream>>>(a);
     }

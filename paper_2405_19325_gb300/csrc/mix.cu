@@ -204,7 +204,7 @@ cudaError_t launch_mix(const MixArgs& a, cudaStream_t stream)
     const int widest = unit * (int)((units + a.slices - 1) / a.slices) + unit;
     const size_t smem = (size_t)widest * sizeof(unsigned long long);
     cudaError_t e =
-        cudaFuncSetAttribute(mix_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        raise_smem_limit(reinterpret_cast<const void*>(mix_kernel), (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid(a.slices, a.B);
     mix_kernel<<<grid, kMixThreads, smem, stream>>>(a);

@@ -407,8 +407,7 @@ template <int DT, int NQ, int CPT>
 cudaError_t launch_impl(const ScanPlan& p, const ScanArgs& a, cudaStream_t stream)
 {
     auto kern = scan_topr_kernel<DT, NQ, CPT>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)p.smem);
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
     kern<<<p.groups * p.parts, kScanThreads, p.smem, stream>>>(a);
     return cudaGetLastError();

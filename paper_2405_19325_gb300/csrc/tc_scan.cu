@@ -298,7 +298,7 @@ cudaError_t tc_launch_nq(const TcPlan& p, const CUtensorMap& tmK, const CUtensor
 {
     auto kern = tc_scan_kernel<NQ>;
     cudaError_t e =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+        raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
     kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
     return cudaGetLastError();

@@ -930,15 +930,14 @@ cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUte
                            const WideArgs& a, cudaStream_t stream)
 {
     if (NM == 256 && p.mb == 2) {
-        cudaError_t e = cudaFuncSetAttribute(tc_wide2_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+        cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_wide2_kernel), (int)p.smem);
         if (e != cudaSuccess) return e;
         tc_wide2_kernel<<<p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ, a);
         return cudaGetLastError();
     }
     auto kern = tc_wide_kernel<NM>;
     cudaError_t e =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+        raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
     kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
     return cudaGetLastError();
@@ -985,8 +984,7 @@ cudaError_t launch_gselect(const GselectArgs& in, cudaStream_t stream)
     while (P2 < a.r) P2 <<= 1;
     a.stage_words = P2 > 16384 ? P2 : 16384;  // at least next_pow2(r): the sort runs there
     const size_t smem = (size_t)a.stage_words * sizeof(uint64_t);
-    cudaError_t e = cudaFuncSetAttribute(gselect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(gselect_kernel), (int)smem);
     if (e != cudaSuccess) return e;
     gselect_kernel<<<a.B, kSelThreads, smem, stream>>>(a);
     return cudaGetLastError();
