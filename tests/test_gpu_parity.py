@@ -381,6 +381,30 @@ def test_wide_batch_keys_stored_cluster_by_cluster(nest):
     run_and_check(nest, K, V, q, p_lm, r, 1 / 16, 0.8, vocab, "bf16", check_rows=rows)
 
 
+def test_wide_batch_massive_exact_ties(nest):
+    """Groups of 256 queries over keys that are exact copies of two integer
+    vectors (two of every three keys are the same vector): every query sees
+    two distances, the r nearest are the r smallest indices among the nearer
+    copies, and the bin of the r-th smallest word holds tens of thousands of
+    words, more than the exact selection stages in shared memory.  Integer
+    values keep the fp32 distances exact, so the lists must match bit for
+    bit.  bf16, d=64, N=100,000 (one pass), B=300, r=64."""
+    g = torch.Generator().manual_seed(41)
+    N, d, B, r, vocab = 100000, 64, 300, 64, 500
+    b0 = torch.randint(-2, 3, (d,), generator=g).float()
+    b1 = b0.clone()
+    b1[0] += 1
+    K = torch.where((torch.arange(N) % 3 == 0)[:, None], b1, b0).to(torch.bfloat16)
+    q = (b0 + torch.randint(-1, 2, (B, d), generator=g).float()).to(torch.bfloat16)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g), dim=1)
+    ds = nest.Datastore(K.cuda(), V.cuda(), vocab)
+    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.close()
+    rows = list(range(0, B, 23)) + [B - 1]
+    run_and_check(nest, K, V, q, p_lm, r, 1 / 8, 0.7, vocab, "bf16", exact=True, check_rows=rows)
+
+
 def test_large_batch_shape_sampled_rows(nest):
     """Large-batch shape: bf16 d=4096, B=512, r=256, clustered keys (N reduced
     to 524,288); the oracle checks 12 query rows spread over the batch."""
