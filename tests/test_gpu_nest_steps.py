@@ -98,11 +98,14 @@ def test_verify_spans_matches_oracle(nest):
     ds.close()
 
 
-@pytest.mark.parametrize("path,B,r,dtype", [("tc_scan_kernel", 4, 64, "bf16"),
-                                             ("tc_wide_kernel", 40, 128, "bf16"),
-                                             ("scan_topr_kernel", 3, 50, "f32")])
-def test_masked_search_skips_used_keys(nest, path, B, r, dtype):
-    K, V, q, p_lm = _case(60000, 256, B, 300, seed=42, dtype=dtype)
+@pytest.mark.parametrize("path,B,r,dtype,N", [("tc_scan_kernel", 4, 64, "bf16", 60000),
+                                               ("tc_wide_kernel", 40, 128, "bf16", 60000),
+                                               ("scan_topr_kernel", 3, 50, "f32", 60000),
+                                               # groups of 256: one pass, then two passes
+                                               ("tc_wide2_kernel", 300, 128, "bf16", 60000),
+                                               ("tc_wide2_kernel", 260, 64, "bf16", 140000)])
+def test_masked_search_skips_used_keys(nest, path, B, r, dtype, N):
+    K, V, q, p_lm = _case(N, 256, B, 300, seed=42, dtype=dtype)
     ds = nest.Datastore(K, V, 300)
     assert ds.search_path(B, r) == path
     mask = ds.new_key_mask()
@@ -111,7 +114,7 @@ def test_masked_search_skips_used_keys(nest, path, B, r, dtype):
     s0, i0 = ds.search(q, r)
     first = int(i0[0, 0])
     ds.mask_keys(mask, max(0, first - 20), 64)
-    bits = torch.rand(60000, generator=g) < 0.2
+    bits = torch.rand(N, generator=g) < 0.2
     ds.mask_keys(mask, 1000, 4000)
     words = mask.cpu().numpy().view(np.uint32)
     for k in np.flatnonzero(bits.numpy()):
@@ -120,12 +123,14 @@ def test_masked_search_skips_used_keys(nest, path, B, r, dtype):
     s, idx = ds.search_masked(q, r, mask)
     torch.cuda.synchronize()
     assert ds.device_status() == 0
-    excl = ((words[np.arange(60000) >> 5] >> (np.arange(60000) & 31)) & 1).astype(bool)
+    excl = ((words[np.arange(N) >> 5] >> (np.arange(N) & 31)) & 1).astype(bool)
     K_np, q_np = synth.to_numpy_raw(K), synth.to_numpy_raw(q)
-    s_or, i_or = oracle.knn_search(K_np, q_np, r, exclude=excl)
+    rows = list(range(0, B, max(1, B // 12))) + [B - 1]
+    s_or, i_or = oracle.knn_search(K_np, q_np[rows], r, exclude=excl)
     i_np = idx.cpu().numpy()
     assert not excl[i_np[i_np >= 0]].any()
-    check_search(s.cpu().numpy(), i_np, s_or, i_or, K_np, q_np, dtype, np.full(B, 60000))
+    check_search(s.cpu().numpy()[rows], i_np[rows], s_or, i_or, K_np, q_np[rows], dtype,
+                 np.full(len(rows), N))
     ds.close()
 
 
