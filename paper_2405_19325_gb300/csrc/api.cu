@@ -169,7 +169,13 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
         WidePlan wp{};
         if (wide_plan_smem(nm, ds->smem_optin, &wp)) {
             wp.groups = (B + nm - 1) / nm;
-            const int64_t target = std::max<int64_t>(65536, 256LL * r);
+            // Sample of about max(65,536, k r) keys, so that at most a
+            // fraction 1/k of the keys survives its r-th distance.  Groups of
+            // 256 queries run a tensor-bound main pass whose epilogue the
+            // survivors slow down (k = 256); smaller batches gain more from a
+            // cheaper sampling pass and selection (k = 64).
+            const int64_t k = nm == 256 ? 256 : 64;
+            const int64_t target = std::max<int64_t>(65536, k * r);
             sp->stride = std::max<int64_t>(1, ds->N / target);
             sp->sample_rows = ds->N / sp->stride;
             sp->single_pass = sp->stride == 1;
