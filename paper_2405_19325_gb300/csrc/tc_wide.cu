@@ -142,15 +142,25 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
     uint32_t* st = stage + lane;
     uint32_t m = 0;
     int n = 0;
+    const float2 kn2 = make_float2(kn, kn), m2 = make_float2(-2.f, -2.f);
 #pragma unroll
     for (int v = 0; v < W / 4; ++v) {
         const float4 qv = *reinterpret_cast<const float4*>(sh.qn + c0 + 4 * v);
         const int4 tv = *reinterpret_cast<const int4*>(sh.thr + c0 + 4 * v);
-        const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
         const int ta[4] = {tv.x, tv.y, tv.z, tv.w};
+        // two columns per packed add / fma (each lane rounds as fmaf would)
+        const float2 d01 = __ffma2_rn(m2,
+                                      make_float2(__uint_as_float(acc[4 * v]),
+                                                  __uint_as_float(acc[4 * v + 1])),
+                                      __fadd2_rn(make_float2(qv.x, qv.y), kn2));
+        const float2 d23 = __ffma2_rn(m2,
+                                      make_float2(__uint_as_float(acc[4 * v + 2]),
+                                                  __uint_as_float(acc[4 * v + 3])),
+                                      __fadd2_rn(make_float2(qv.z, qv.w), kn2));
+        const float da[4] = {d01.x, d01.y, d23.x, d23.y};
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            const float dist = fmaf(-2.f, __uint_as_float(acc[4 * v + k]), qa[k] + kn);
+            const float dist = da[k];
             const bool b = valid && __float_as_int(dist) <= ta[k];
             m |= (b ? 1u : 0u) << (4 * v + k);
             if (staging) {
