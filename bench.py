@@ -283,16 +283,17 @@ def run_reference(args, w, world, rank):
     print(json.dumps(line), flush=True)
 
 
-# DRAM bytes (read + write) per launch of the dominant kernel, from the ncu
-# capture summarised in profiles/tc_scan_decode_d4096_B4.md: 65,536-key case
-# scaled to the default 1,048,576 keys (reads x16, per-CTA writes unscaled).
-# Only valid for that kernel version on the default decode workload.
+# DRAM bytes (read + write) per launch of the dominant kernel, from one ncu
+# capture (dram__bytes_read.sum + dram__bytes_write.sum) of tc_scan_kernel on
+# a 65,536-key case, scaled to the default 1,048,576 keys (reads x16, per-CTA
+# writes unscaled).  Only valid for that kernel version on the default decode
+# workload.
 DECODE_TC_SCAN_TRAFFIC = 537.278464e6 * 16 + 3.055104e6
 
-# Same for the large-batch main pass, from profiles/tc_wide2_large_batch_B512.md:
-# the 262,144-key case scaled by 16 to the default 4,194,304 keys (key reads
-# and, with the sample size fixed at 65,536 keys, survivor writes both grow
-# with N).  Only valid for that kernel version on the default large batch.
+# Same for the large-batch main pass (tc_wide2_kernel): a 262,144-key capture
+# scaled by 16 to the default 4,194,304 keys (key reads and, with the sample
+# size fixed at 65,536 keys, survivor writes both grow with N).  Only valid
+# for that kernel version on the default large batch.
 LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.310617e9 + 28.610304e6) * 16
 
 
