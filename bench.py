@@ -294,7 +294,7 @@ DECODE_TC_SCAN_TRAFFIC = 537.278464e6 * 16 + 3.055104e6
 # scaled by 16 to the default 4,194,304 keys (key reads and, with the sample
 # size fixed at 65,536 keys, survivor writes both grow with N).  Only valid
 # for that kernel version on the default large batch.
-LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.310617e9 + 28.610304e6) * 16
+LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.323294e9 + 28.291072e6) * 16
 
 
 def dram_traffic(w, args, kernel):
