@@ -738,17 +738,21 @@ struct GselShared {
 };
 
 // Copies the real words of list[0, n) that `keep` accepts into stage[]
-// (order not kept; the caller sorts).  Returns after a barrier.
+// (order not kept; the caller sorts).  Returns after a barrier.  The loop
+// runs while the warp's first element is in range, so all 32 lanes make the
+// same number of trips and meet at every ballot and shuffle inside it (a
+// lane leaving early for the closing barrier would leave the others waiting
+// at the ballot forever).
 template <class Keep>
 __device__ __forceinline__ void gsel_copy(const uint64_t* list, int n, uint64_t* stage,
                                           GselShared& sh, int tid, Keep keep)
 {
     const int lane = tid & 31;
-    for (int base = tid; base < n; base += kGselUnroll * kSelThreads) {
+    for (int wbase = tid - lane; wbase < n; wbase += kGselUnroll * kSelThreads) {
         uint64_t v[kGselUnroll];
 #pragma unroll
         for (int u = 0; u < kGselUnroll; ++u) {
-            const int j = base + u * kSelThreads;
+            const int j = wbase + lane + u * kSelThreads;
             v[u] = j < n ? list[j] : kNoCandidate;
         }
 #pragma unroll

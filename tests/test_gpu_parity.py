@@ -359,6 +359,42 @@ def test_two_tile_wide_kernel_edges(nest, N, d, B, r):
     run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 900, "bf16", check_rows=rows)
 
 
+@pytest.mark.parametrize("N,r,masked", [
+    (119, 4096, True),    # r above N, every list shorter than one warp's stride
+    (119, 32, False),
+    (8269, 64, False),    # 8269 = 8192 + 77: the last copy trip splits a warp
+])
+def test_wide_batch_list_lengths_that_split_a_warp(nest, N, r, masked):
+    """Batches over a datastore small enough for one pass: each query's list
+    holds N words, and when N mod 8192 is below 1024 and not a multiple of 32
+    some warp of the selection kernel has lanes with and lanes without a
+    word on the last copy trip.  bf16, d=72, B=100."""
+    B, d, vocab = 100, 72, 500
+    K, V, q, p_lm = _random_case(N, d, B, vocab, "bf16", seed=N + r)
+    ds = nest.Datastore(K.cuda(), V.cuda(), vocab)
+    assert ds.search_path(B, r) == "tc_wide_kernel"
+    if not masked:
+        ds.close()
+        run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, vocab, "bf16",
+                      check_rows=list(range(0, B, 11)) + [B - 1])
+        return
+    excl = np.zeros(N, bool)
+    excl[30:47] = True
+    excl[::7] = True
+    words = np.zeros((N + 31) // 32, dtype=np.uint32)
+    for k in np.flatnonzero(excl):
+        words[k >> 5] |= np.uint32(1 << (k & 31))
+    mask = torch.from_numpy(words.view(np.int32)).cuda()
+    s, idx = ds.search_masked(q.cuda(), r, mask)
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    K_np, q_np = _np(K), _np(q)
+    s_or, i_or = oracle.knn_search(K_np, q_np, r, exclude=excl)
+    check_search(s.cpu().numpy(), idx.cpu().numpy(), s_or, i_or, K_np, q_np, "bf16",
+                 np.full(B, N - int(excl.sum())))
+    ds.close()
+
+
 def test_wide_batch_keys_stored_cluster_by_cluster(nest):
     """Keys stored cluster after cluster (as a datastore built document by
     document would be): each query's main-pass survivors come from the one or

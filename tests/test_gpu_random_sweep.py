@@ -1,0 +1,179 @@
+"""Seeded random sweep of search shapes against the fp64 oracle.
+
+The hand-picked cases elsewhere pin each edge on purpose; this sweep draws
+shapes at random to reach combinations nobody picked: any element type, row
+width, batch, r, datastore size, key layout, ragged segments and key masks,
+with the search path following from the shape.  The cases are drawn once
+from a fixed seed, so every run sees the same 60 shapes and a failure names
+its case.  Each case is held to the same rules as the other parity tests
+(neighbour sets up to ties at the r-th distance, distances within the fp32
+bound, Eq. 2 / Eq. 3 on the GPU's own neighbours); integer layouts must
+match bit for bit.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from parity import check_mix, check_mix_end_to_end, check_search
+
+pytestmark = pytest.mark.gpu
+
+N_CASES = 60
+# keep the oracle's work per case bounded: checked rows x N x d
+MAX_ORACLE_WORK = 2.0e9
+BATCHES = [1, 2, 3, 4, 5, 8, 13, 16, 17, 33, 40, 64, 100, 200, 255, 256, 257, 300, 511, 512, 600]
+RS = [1, 2, 7, 32, 64, 100, 255, 256, 257, 1000, 1024, 2048, 4096]
+WIDTHS = [8, 16, 24, 40, 64, 72, 128, 136, 256, 520, 1024, 2048, 4096]
+LAYOUTS = ["clustered", "sorted_clusters", "uniform", "integer"]
+
+
+def _draw_cases():
+    rng = np.random.default_rng(2405_19325)
+    cases = []
+    while len(cases) < N_CASES:
+        dtype = "bf16" if rng.random() < 0.75 else "f32"
+        esize = 2 if dtype == "bf16" else 4
+        d = int(rng.choice([w for w in WIDTHS if w * esize <= 16384 and (w * esize) % 16 == 0]))
+        B = int(rng.choice(BATCHES))
+        r = int(rng.choice(RS))
+        ragged = bool(rng.random() < 0.25)
+        masked = bool(rng.random() < 0.3)
+        layout = str(rng.choice(LAYOUTS))
+        # log-uniform datastore size; three draws in ten above the threshold
+        # sample (65,536 keys or more) so that batched searches take two passes
+        lo, hi = (60000, 700000) if rng.random() < 0.3 else (1, 400000)
+        N = int(np.exp(rng.uniform(np.log(lo), np.log(hi))))
+        rows = min(B, 10)
+        if rows * N * d > MAX_ORACLE_WORK or N * d > 2.5e8:
+            continue
+        cases.append(dict(dtype=dtype, d=d, B=B, r=r, N=N, ragged=ragged, masked=masked,
+                          layout=layout, seed=int(rng.integers(1 << 30))))
+    return cases
+
+
+CASES = _draw_cases()
+
+
+def _case_id(c):
+    return (f"{c['dtype']}-N{c['N']}-d{c['d']}-B{c['B']}-r{c['r']}-{c['layout']}"
+            + ("-ragged" if c["ragged"] else "") + ("-masked" if c["masked"] else ""))
+
+
+@pytest.fixture(scope="module")
+def nest():
+    from paper_2405_19325_gb300 import build as nest_build
+    nest_build.build()
+    import paper_2405_19325_gb300 as pkg
+    pkg.load_library()
+    return pkg
+
+
+def _inputs(c, vocab):
+    """Keys, values, queries, p_LM, segment offsets and excluded keys of a case."""
+    N, d, B = c["N"], c["d"], c["B"]
+    g = torch.Generator().manual_seed(c["seed"])
+    nc = int(torch.randint(2, 65, (1,), generator=g))
+    if c["layout"] == "integer":
+        # a few integer base vectors plus small integer offsets: fp32 distances exact,
+        # many exact ties
+        base = torch.randint(-2, 3, (nc, d), generator=g).float()
+        K = base[torch.randint(0, nc, (N,), generator=g)] \
+            + (torch.rand(N, d, generator=g) < 0.05).float()
+        q = base[torch.randint(0, nc, (B,), generator=g)] \
+            + torch.randint(-1, 2, (B, d), generator=g).float()
+    else:
+        cen = torch.randn(nc, d, generator=g)
+        if c["layout"] == "uniform":
+            K = torch.randn(N, d, generator=g)
+        elif c["layout"] == "sorted_clusters":
+            K = cen[torch.arange(N) * nc // max(N, 1)] + 0.3 * torch.randn(N, d, generator=g)
+        else:
+            K = cen[torch.randint(0, nc, (N,), generator=g)] + 0.3 * torch.randn(N, d, generator=g)
+        q = cen[torch.randint(0, nc, (B,), generator=g)] + 0.3 * torch.randn(B, d, generator=g)
+    dt = synth.torch_dtype(c["dtype"])
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g) * 2, dim=1)
+    seg_off = None
+    if c["ragged"]:
+        cuts = torch.sort(torch.randint(0, N + 1, (B - 1,), generator=g)).values
+        seg_off = torch.cat([torch.zeros(1, dtype=torch.int64), cuts.to(torch.int64),
+                             torch.full((1,), N, dtype=torch.int64)])
+        if B > 2:  # one empty segment in the middle
+            seg_off[B // 2 + 1] = seg_off[B // 2]
+            seg_off = torch.cummax(seg_off, 0).values
+    excl = None
+    if c["masked"]:
+        excl = (torch.rand(N, generator=g) < 0.15).numpy()
+        a = int(torch.randint(0, N, (1,), generator=g))
+        excl[a:a + max(1, N // 7)] = True          # one used span of keys
+    return K.to(dt), V, q.to(dt), p_lm, seg_off, excl
+
+
+def _mask_words(excl):
+    N = excl.size
+    words = np.zeros((N + 31) // 32, dtype=np.uint32)
+    k = np.flatnonzero(excl)
+    np.bitwise_or.at(words, k >> 5, (np.uint32(1) << (k & 31).astype(np.uint32)))
+    return torch.from_numpy(words.view(np.int32))
+
+
+@pytest.mark.parametrize("c", CASES, ids=[_case_id(c) for c in CASES])
+def test_random_shape(nest, c):
+    vocab = 700
+    N, d, B, r, dtype = c["N"], c["d"], c["B"], c["r"], c["dtype"]
+    K, V, q, p_lm, seg_off, excl = _inputs(c, vocab)
+    dev = torch.device("cuda")
+    ds = nest.Datastore(K.to(dev), V.to(dev), vocab)
+    qd = q.to(dev)
+    so_d = seg_off.to(dev) if seg_off is not None else None
+    mu, lam = 1 / np.sqrt(d), 0.75
+    # full scans: a spread of rows; ragged: every row (each scans only its segment)
+    rows = list(range(B)) if c["ragged"] else sorted(set(range(0, B, max(1, B // 9))) | {B - 1})
+    K_np, V_np = synth.to_numpy_raw(K), V.numpy()
+    q_np = synth.to_numpy_raw(q)[rows]
+    p_lm_np = p_lm.numpy()[rows]
+    so_np = seg_off.numpy() if seg_off is not None else None
+    exact = c["layout"] == "integer"
+    if excl is None:
+        out = ds.step(qd, r, p_lm.to(dev), mu, lam, seg_off=so_d, want_p_knn=True)
+        torch.cuda.synchronize()
+        assert ds.device_status() == 0
+        s_g, i_g = out["s"].cpu().numpy()[rows], out["idx"].cpu().numpy()[rows]
+        ref = oracle.knn_step(K_np, V_np, q_np, r, p_lm_np, mu, lam, vocab, seg_off=so_np)
+        counts = (np.full(B, N) if so_np is None else so_np[1:] - so_np[:-1])[rows]
+        matched = check_search(s_g, i_g, ref["s"], ref["idx"], K_np, q_np, dtype, counts,
+                               exact=exact)
+        p_m = out["p_m"].cpu().numpy()[rows]
+        check_mix(p_m, s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
+                  p_knn_gpu=out["p_knn"].cpu().numpy()[rows])
+        check_mix_end_to_end(p_m, ref["p_m"], matched)
+    else:
+        mask = _mask_words(excl).to(dev)
+        s, idx = ds.search_masked(qd, r, mask, seg_off=so_d)
+        torch.cuda.synchronize()
+        assert ds.device_status() == 0
+        i_all = idx.cpu().numpy()
+        assert not excl[i_all[i_all >= 0]].any(), "a masked key was returned"
+        s_or, i_or = oracle.knn_search(K_np, q_np, r, seg_off=so_np, exclude=excl)
+        if so_np is None:
+            counts = np.full(len(rows), N - int(excl.sum()))
+        else:
+            counts = np.array([int(so_np[b + 1] - so_np[b] - excl[so_np[b]:so_np[b + 1]].sum())
+                               for b in range(B)])[rows]
+        check_search(s.cpu().numpy()[rows], i_all[rows], s_or, i_or, K_np, q_np, dtype, counts,
+                     exact=exact)
+    ds.close()
+
+
+def test_sweep_reaches_every_search_path(nest):
+    """The drawn shapes run every distance-scan kernel the library has."""
+    seen = set()
+    V = torch.zeros(64, dtype=torch.int32, device="cuda")
+    for c in CASES:
+        K = torch.zeros(64, c["d"], dtype=synth.torch_dtype(c["dtype"]), device="cuda")
+        ds = nest.Datastore(K, V, 10)
+        seen.add(ds.search_path(c["B"], c["r"], ragged=c["ragged"]))
+        ds.close()
+    assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel", "scan_topr_kernel"}, seen
