@@ -4,11 +4,18 @@ The hand-picked cases elsewhere pin each edge on purpose; this sweep draws
 shapes at random to reach combinations nobody picked: any element type, row
 width, batch, r, datastore size, key layout, ragged segments and key masks,
 with the search path following from the shape.  The cases are drawn once
-from a fixed seed, so every run sees the same 60 shapes and a failure names
+from a fixed seed, so every run sees the same shapes and a failure names
 its case.  Each case is held to the same rules as the other parity tests
 (neighbour sets up to ties at the r-th distance, distances within the fp32
 bound, Eq. 2 / Eq. 3 on the GPU's own neighbours); integer layouts must
 match bit for bit.
+
+A second set draws every size from values next to the ones the kernels
+branch on (tile and warp multiples, the 8,192-word copy stride of the
+selection, the 65,536-key threshold sample, the query-group sizes, list
+lengths around 1,024) and goes through each public entry point in turn:
+the device step, the host-buffer step, search + Eq. 4 + the Eq. 5 / Eq. 6
+decision, and the masked search.
 """
 import numpy as np
 import pytest
@@ -55,10 +62,46 @@ def _draw_cases():
 
 CASES = _draw_cases()
 
+EDGE_N = [1, 2, 31, 33, 127, 128, 129, 255, 257, 1023, 1024, 1025, 1057, 8191, 8192, 8193,
+          8269, 9215, 16447, 65535, 65536, 65537, 65599, 131071, 131073, 196705, 262145]
+EDGE_B = [1, 2, 3, 4, 5, 15, 16, 17, 31, 33, 63, 64, 65, 127, 128, 129, 255, 256, 257, 383,
+          384, 511, 512, 513]
+EDGE_R = [1, 2, 31, 32, 33, 255, 256, 257, 511, 512, 513, 1023, 1024, 1025, 2047, 2048, 4095, 4096]
+EDGE_D = {"bf16": [8, 56, 64, 72, 120, 128, 136, 1016, 4096, 8192],
+          "f32": [4, 60, 64, 68, 1020, 4096]}
+ENTRIES = ["step", "host", "rrc_decide", "masked"]
+N_EDGE = 60
+
+
+def _draw_edge_cases():
+    rng = np.random.default_rng(7_2405)
+    cases = []
+    while len(cases) < N_EDGE:
+        dtype = "bf16" if rng.random() < 0.75 else "f32"
+        d = int(rng.choice(EDGE_D[dtype]))
+        B = int(rng.choice(EDGE_B))
+        r = int(rng.choice(EDGE_R))
+        N = int(rng.choice(EDGE_N))
+        entry = ENTRIES[len(cases) % len(ENTRIES)]
+        ragged = entry != "rrc_decide" and bool(rng.random() < 0.2)
+        layout = str(rng.choice(LAYOUTS))
+        rows = B if ragged else min(B, 10)
+        if rows * N * d > MAX_ORACLE_WORK or N * d > 2.5e8:
+            continue
+        cases.append(dict(dtype=dtype, d=d, B=B, r=r, N=N, ragged=ragged,
+                          masked=entry == "masked", layout=layout, entry=entry,
+                          seed=int(rng.integers(1 << 30))))
+    return cases
+
+
+EDGE_CASES = _draw_edge_cases()
+
 
 def _case_id(c):
+    entry = c.get("entry")
     return (f"{c['dtype']}-N{c['N']}-d{c['d']}-B{c['B']}-r{c['r']}-{c['layout']}"
-            + ("-ragged" if c["ragged"] else "") + ("-masked" if c["masked"] else ""))
+            + ("-ragged" if c["ragged"] else "")
+            + (f"-{entry}" if entry else ("-masked" if c["masked"] else "")))
 
 
 @pytest.fixture(scope="module")
@@ -121,6 +164,15 @@ def _mask_words(excl):
 
 @pytest.mark.parametrize("c", CASES, ids=[_case_id(c) for c in CASES])
 def test_random_shape(nest, c):
+    _run_case(nest, c)
+
+
+@pytest.mark.parametrize("c", EDGE_CASES, ids=[_case_id(c) for c in EDGE_CASES])
+def test_boundary_shape(nest, c):
+    _run_case(nest, c)
+
+
+def _run_case(nest, c):
     vocab = 700
     N, d, B, r, dtype = c["N"], c["d"], c["B"], c["r"], c["dtype"]
     K, V, q, p_lm, seg_off, excl = _inputs(c, vocab)
@@ -136,19 +188,46 @@ def test_random_shape(nest, c):
     p_lm_np = p_lm.numpy()[rows]
     so_np = seg_off.numpy() if seg_off is not None else None
     exact = c["layout"] == "integer"
-    if excl is None:
-        out = ds.step(qd, r, p_lm.to(dev), mu, lam, seg_off=so_d, want_p_knn=True)
-        torch.cuda.synchronize()
+    entry = c.get("entry", "masked" if excl is not None else "step")
+    counts = (np.full(B, N) if so_np is None else so_np[1:] - so_np[:-1])[rows]
+    if entry in ("step", "host"):
+        if entry == "step":
+            out = ds.step(qd, r, p_lm.to(dev), mu, lam, seg_off=so_d, want_p_knn=True)
+            torch.cuda.synchronize()
+            p_knn = out["p_knn"].cpu().numpy()[rows]
+        else:
+            out = ds.step_host(q.pin_memory(), r, p_lm.pin_memory(), mu, lam,
+                               seg_off_host=seg_off)
+            p_knn = None
         assert ds.device_status() == 0
         s_g, i_g = out["s"].cpu().numpy()[rows], out["idx"].cpu().numpy()[rows]
         ref = oracle.knn_step(K_np, V_np, q_np, r, p_lm_np, mu, lam, vocab, seg_off=so_np)
-        counts = (np.full(B, N) if so_np is None else so_np[1:] - so_np[:-1])[rows]
         matched = check_search(s_g, i_g, ref["s"], ref["idx"], K_np, q_np, dtype, counts,
                                exact=exact)
         p_m = out["p_m"].cpu().numpy()[rows]
-        check_mix(p_m, s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
-                  p_knn_gpu=out["p_knn"].cpu().numpy()[rows])
+        check_mix(p_m, s_g, i_g, V_np, p_lm_np, mu, lam, vocab, p_knn_gpu=p_knn)
         check_mix_end_to_end(p_m, ref["p_m"], matched)
+    elif entry == "rrc_decide":
+        alpha, tau, delta = 0.3, 0.1, 0.5
+        s, idx = ds.search(qd, r, seg_off=so_d)
+        p_m, lam_t = ds.mix_rrc(s, idx, p_lm.to(dev), mu, alpha, tau)
+        o = ds.decide(p_m, s, idx, lam_t, delta)
+        torch.cuda.synchronize()
+        assert ds.device_status() == 0
+        s_g, i_g = s.cpu().numpy()[rows], idx.cpu().numpy()[rows]
+        s_or, i_or = oracle.knn_search(K_np, q_np, r, seg_off=so_np)
+        check_search(s_g, i_g, s_or, i_or, K_np, q_np, dtype, counts, exact=exact)
+        lam_g = lam_t.cpu().numpy()[rows]
+        np.testing.assert_allclose(lam_g, oracle.rrc(s_g.astype(np.float64), i_g, alpha, tau),
+                                   rtol=0, atol=1e-6)
+        p_m_g = p_m.cpu().numpy()[rows]
+        check_mix(p_m_g, s_g, i_g, V_np, p_lm_np, mu, None, vocab, lam_gpu=lam_g)
+        tok, pmax, key, use = oracle.decide(p_m_g.astype(np.float64), s_g, i_g, V_np,
+                                            lam_g.astype(np.float64), delta)
+        assert o["token"].cpu().numpy()[rows].tolist() == tok.tolist()
+        np.testing.assert_array_equal(o["p_max"].cpu().numpy()[rows].astype(np.float64), pmax)
+        assert o["span_key"].cpu().numpy()[rows].tolist() == key.tolist()
+        assert o["use_span"].cpu().numpy()[rows].tolist() == use.tolist()
     else:
         mask = _mask_words(excl).to(dev)
         s, idx = ds.search_masked(qd, r, mask, seg_off=so_d)
@@ -171,7 +250,7 @@ def test_sweep_reaches_every_search_path(nest):
     """The drawn shapes run every distance-scan kernel the library has."""
     seen = set()
     V = torch.zeros(64, dtype=torch.int32, device="cuda")
-    for c in CASES:
+    for c in CASES + EDGE_CASES:
         K = torch.zeros(64, c["d"], dtype=synth.torch_dtype(c["dtype"]), device="cuda")
         ds = nest.Datastore(K, V, 10)
         seen.add(ds.search_path(c["B"], c["r"], ragged=c["ragged"]))
