@@ -27,7 +27,7 @@ from parity import check_mix, check_mix_end_to_end, check_search
 
 pytestmark = pytest.mark.gpu
 
-N_CASES = 60
+N_CASES = 100
 # keep the oracle's work per case bounded: checked rows x N x d
 MAX_ORACLE_WORK = 2.0e9
 BATCHES = [1, 2, 3, 4, 5, 8, 13, 16, 17, 33, 40, 64, 100, 200, 255, 256, 257, 300, 511, 512, 600]
@@ -70,7 +70,7 @@ EDGE_R = [1, 2, 31, 32, 33, 255, 256, 257, 511, 512, 513, 1023, 1024, 1025, 2047
 EDGE_D = {"bf16": [8, 56, 64, 72, 120, 128, 136, 1016, 4096, 8192],
           "f32": [4, 60, 64, 68, 1020, 4096]}
 ENTRIES = ["step", "host", "rrc_decide", "masked"]
-N_EDGE = 60
+N_EDGE = 100
 
 
 def _draw_edge_cases():
