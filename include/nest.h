@@ -294,6 +294,8 @@ NEST_API nest_status_t nest_knn_decide(nest_datastore_t* ds, const float* p_m, c
  *                     the first position whose acceptance is at most 1/2)
  *   n_accept_out[j] = number of leading accepted positions of span j
  *
+ * 1 <= rows <= 65535 and 1 <= spans <= 65535; a span may be empty
+ * (span_off[j] == span_off[j+1], n_accept = 0).
  * gamma in (0, 1] is the relaxation factor.  A draft token outside
  * [0, vocab) is rejected and recorded as NEST_ERR_VALUE_RANGE; bad span
  * offsets give n_accept = 0 and NEST_ERR_INVALID_ARG in the device status.

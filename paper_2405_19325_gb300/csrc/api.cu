@@ -906,7 +906,7 @@ nest_status_t nest_verify_spans(nest_datastore_t* ds, const float* p_m, const in
 {
     if (!ds || !p_m || !draft || !span_off || !ratio_out || !accept_out || !n_accept_out)
         return NEST_ERR_INVALID_ARG;
-    if (rows < 1 || rows > kMaxB || spans < 1 || spans > rows || !(gamma > 0.f))
+    if (rows < 1 || rows > kMaxB || spans < 1 || spans > kMaxB || !(gamma > 0.f))
         return NEST_ERR_INVALID_ARG;
     if (!aligned(p_m, 4) || !aligned(draft, 4) || !aligned(span_off, 4) || !aligned(ratio_out, 4) ||
         !aligned(accept_out, 4) || !aligned(n_accept_out, 4))

@@ -256,3 +256,147 @@ def test_sweep_reaches_every_search_path(nest):
         seen.add(ds.search_path(c["B"], c["r"], ragged=c["ragged"]))
         ds.close()
     assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel", "scan_topr_kernel"}, seen
+
+
+# ---------------------------------------------------------------- Eq. 7 verification and masking
+
+VOCABS = [1, 2, 3, 7, 31, 1000, 4097, 32000, 50257, 128256]
+P_KINDS = ["peaked", "flat", "one_hot", "tied_max", "with_zero_rows"]
+GAMMAS = [1.0, 0.5, 0.1, 1e-3, 1e-6]
+
+
+def _draw_verify_cases(n=40):
+    rng = np.random.default_rng(7_7)
+    cases = []
+    while len(cases) < n:
+        vocab = int(rng.choice(VOCABS))
+        rows = int(np.exp(rng.uniform(0, np.log(3000))))
+        if rows * vocab > 3e7:
+            continue
+        cases.append(dict(vocab=vocab, rows=rows, kind=str(rng.choice(P_KINDS)),
+                          gamma=float(rng.choice(GAMMAS)), spans=int(rng.integers(1, 65)),
+                          seed=int(rng.integers(1 << 30))))
+    return cases
+
+
+VERIFY_CASES = _draw_verify_cases()
+
+
+def _verify_inputs(c):
+    g = torch.Generator().manual_seed(c["seed"])
+    rows, vocab = c["rows"], c["vocab"]
+    kind = c["kind"]
+    if kind == "flat":
+        p = torch.softmax(torch.randn(rows, vocab, generator=g) * 0.1, dim=1)
+    elif kind == "one_hot":
+        p = torch.zeros(rows, vocab)
+        p[torch.arange(rows), torch.randint(0, vocab, (rows,), generator=g)] = 1.0
+    else:
+        p = torch.softmax(torch.randn(rows, vocab, generator=g) * 8, dim=1)
+    if kind == "tied_max" and vocab > 1:
+        # the two largest entries of every row set equal
+        top2 = torch.topk(p, 2, dim=1)
+        p[torch.arange(rows), top2.indices[:, 1]] = top2.values[:, 0]
+    if kind == "with_zero_rows":
+        p[torch.rand(rows, generator=g) < 0.2] = 0.0
+    top = p.argmax(1).to(torch.int32)
+    other = torch.randint(0, vocab, (rows,), generator=g, dtype=torch.int32)
+    if vocab > 1:
+        second = torch.topk(p, 2, dim=1).indices[:, 1].to(torch.int32)
+    else:
+        second = top
+    u = torch.rand(rows, generator=g)
+    draft = torch.where(u < 0.6, top, torch.where(u < 0.8, second, other))
+    cuts = torch.sort(torch.randint(0, rows + 1, (c["spans"] - 1,), generator=g)).values
+    off = torch.cat([torch.zeros(1, dtype=torch.int32), cuts.to(torch.int32),
+                     torch.full((1,), rows, dtype=torch.int32)])
+    return p.contiguous(), draft, off
+
+
+def _verify_id(c):
+    return f"V{c['vocab']}-rows{c['rows']}-spans{c['spans']}-{c['kind']}-g{c['gamma']:g}"
+
+
+@pytest.mark.parametrize("c", VERIFY_CASES, ids=[_verify_id(c) for c in VERIFY_CASES])
+def test_verify_random(nest, c):
+    """Eq. 7 on random spans (empty spans included) against the oracle: the
+    ratio within fp32 rounding, the acceptance flags exactly except where
+    min(1, ratio) lies within rounding of 1/2, and each span's accepted
+    prefix following the GPU's own flags."""
+    p, draft, off = _verify_inputs(c)
+    dev = torch.device("cuda")
+    K = torch.randn(64, 16, device=dev)
+    ds = nest.Datastore(K, torch.zeros(64, dtype=torch.int32, device=dev), c["vocab"])
+    o = ds.verify(p.to(dev), draft.to(dev), off.to(dev), c["gamma"])
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    ratio, acc, n_acc = oracle.verify(p.numpy().astype(np.float64), draft.numpy(), off.numpy(),
+                                      c["gamma"])
+    g_ratio = o["ratio"].cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(g_ratio, ratio, rtol=2e-6, atol=0)
+    g_acc = o["accept"].cpu().numpy()
+    near = np.abs(np.minimum(ratio, 1.0) - 0.5) <= 1e-6
+    assert np.array_equal(g_acc[~near], acc[~near])
+    g_n = o["n_accept"].cpu().numpy()
+    so = off.numpy()
+    for j in range(len(so) - 1):
+        run = 0
+        while so[j] + run < so[j + 1] and g_acc[so[j] + run]:
+            run += 1
+        assert g_n[j] == run, f"span {j}"
+    if not near.any():
+        assert g_n.tolist() == n_acc.tolist()
+    ds.close()
+
+
+def _draw_mask_cases(n=30):
+    rng = np.random.default_rng(7_31)
+    cases = []
+    for _ in range(n):
+        N = int(np.exp(rng.uniform(0, np.log(2_000_000))))
+        spans = []
+        for _ in range(int(rng.integers(1, 9))):
+            kind = rng.integers(0, 4)
+            if kind == 0:      # empty span
+                first, count = int(rng.integers(0, N + 1)), 0
+            elif kind == 1:    # ends at the last key
+                count = int(rng.integers(1, N + 1))
+                first = N - count
+            elif kind == 2:    # starts on a word boundary
+                first = int(rng.integers(0, N // 32 + 1)) * 32
+                first = min(first, N - 1)
+                count = int(rng.integers(1, min(N - first, 200) + 1))
+            else:
+                first = int(rng.integers(0, N))
+                count = int(rng.integers(1, min(N - first, 5000) + 1))
+            spans.append((first, count))
+        cases.append(dict(N=N, spans=spans))
+    return cases
+
+
+MASK_CASES = _draw_mask_cases()
+
+
+@pytest.mark.parametrize("c", MASK_CASES, ids=[f"N{c['N']}-{len(c['spans'])}spans" for c in MASK_CASES])
+def test_mask_keys_random(nest, c):
+    """Sec. 3.4 masking: the bits nest_mask_keys sets over random runs of
+    keys (empty runs, runs ending at the last key, runs on and off word
+    boundaries, overlapping runs) equal the union of the runs."""
+    N = c["N"]
+    dev = torch.device("cuda")
+    K = torch.zeros(N, 4, device=dev)
+    ds = nest.Datastore(K, torch.zeros(N, dtype=torch.int32, device=dev), 10)
+    mask = ds.new_key_mask()
+    want = np.zeros(N, bool)
+    for first, count in c["spans"]:
+        ds.mask_keys(mask, first, count)
+        want[first:first + count] = True
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    words = mask.cpu().numpy().view(np.uint32)
+    got = ((words[np.arange(N) >> 5] >> (np.arange(N) & 31)) & 1).astype(bool)
+    assert np.array_equal(got, want)
+    tail = N % 32
+    if tail:
+        assert words[-1] >> np.uint32(tail) == 0, "bits past the last key"
+    ds.close()
