@@ -104,6 +104,23 @@ NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_
                                      int32_t ragged);
 
 /*
+ * Whether searches with groups of 256 queries run on CTA pairs (search
+ * path 4 of nest_search_path) or on single CTAs with two key tiles per
+ * pipeline stage (path 3, the default).  Both return the same neighbours.
+ * A pair splits each 256-key tile over two SMs and double-buffers its
+ * accumulators; with one query group it runs as fast as path 3, but with
+ * several groups their pairs drift apart and read the same keys from DRAM
+ * again (1.46 times the key bytes at 1M keys and B = 512 on a GB300,
+ * against 1.10 for path 3), so path 3 stays the default.  Pairs need two
+ * CTAs of about 220 KiB of shared memory each on the two SMs of one TPC at
+ * the same time; on = 1 where the device cannot place them returns
+ * NEST_ERR_UNSUPPORTED and changes nothing.  Host only; takes effect from
+ * the next search, which may need more scratch than nest_datastore_reserve
+ * set aside.
+ */
+NEST_API nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t on);
+
+/*
  * r-nearest-neighbour search (Sec. 2.2; Sec. 3.1 second stage; App. A).
  *
  *   q        B x d queries, the datastore's element type, 16-byte aligned.
@@ -329,6 +346,9 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
  *      thresholds (bf16 keys, more queries than one CTA keeps lists for)
  *   3  the same with two 128-key tiles per pipeline stage (groups of 256
  *      queries, when three 64 KiB stages fit in shared memory)
+ *   4  the same on CTA pairs (groups of 256 queries, 256-key tiles split
+ *      over two SMs, double-buffered accumulators), after
+ *      nest_datastore_use_cta_pairs(ds, 1)
  * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
  */
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,

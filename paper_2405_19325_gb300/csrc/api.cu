@@ -26,6 +26,8 @@ struct nest_datastore {
     int num_sms = 1;
     size_t smem_optin = 0;
     bool tc = false;         // bf16 keys with a TMA tensor map: tensor-core scan
+    bool pairs_ok = false;   // the device can place the wide kernel's CTA pairs
+    bool pairs = false;      // ... and searches use them
     CUtensorMap keys_map;  // TMA map of K (type is 64-byte aligned)
     float* knorm = nullptr;  // owned: ||k_i||^2, N floats
     int* status = nullptr;   // owned: device status word
@@ -167,7 +169,7 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
     if (sp->tc && !ragged && sp->groups > 1) {
         const int nm = B >= 256 ? 256 : std::max(16, ceil_pow2(B));
         WidePlan wp{};
-        if (wide_plan_smem(nm, ds->smem_optin, &wp)) {
+        if (wide_plan_smem(nm, ds->smem_optin, ds->pairs, &wp)) {
             wp.groups = (B + nm - 1) / nm;
             // Sample of about max(65,536, k r) keys, so that at most a
             // fraction 1/k of the keys survives its r-th distance.  Groups of
@@ -180,9 +182,11 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             sp->sample_rows = ds->N / sp->stride;
             sp->single_pass = sp->stride == 1;
             sp->wps = wp;
-            sp->wps.parts = choose_parts(wp.groups, sp->sample_rows, ds->num_sms, false);
+            // a CTA pair takes two SMs
+            const int slots = wp.pair ? ds->num_sms / 2 : ds->num_sms;
+            sp->wps.parts = choose_parts(wp.groups, sp->sample_rows, slots, false);
             sp->wpm = wp;
-            sp->wpm.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
+            sp->wpm.parts = choose_parts(wp.groups, ds->N, slots, false);
             sp->cap_s = sp->sample_rows;
             const int64_t expect = (ds->N * (int64_t)r + sp->sample_rows - 1) / sp->sample_rows;
             // Main-pass lists hold 8x the expected survivors plus what the
@@ -397,7 +401,9 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     cudaError_t e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * 2 * (size_t)B, stream);
     if (e != cudaSuccess) return from_cuda(e);
     CUtensorMap qmap;
-    if (!encode_bf16_rows(&qmap, q, B, ds->d, sp.wpm.nm, false)) return NEST_ERR_CUDA;
+    // a CTA of a pair stages half of the group's queries
+    if (!encode_bf16_rows(&qmap, q, B, ds->d, sp.wpm.pair ? sp.wpm.nm / 2 : sp.wpm.nm, false))
+        return NEST_ERR_CUDA;
 
     WideArgs wa{};
     wa.knorm = ds->knorm;
@@ -688,6 +694,8 @@ nest_status_t nest_datastore_create(const void* K, const int32_t* V, int64_t N, 
     // Tensor-core scan: bf16 keys whose row indices fit TMA's 32-bit coordinates.
     if (dtype == NEST_BF16 && N <= (int64_t)0x7FFFFF00)
         ds->tc = encode_bf16_rows(&ds->keys_map, K, N, d, kTcTileKeys, true);
+    ds->pairs_ok = ds->tc && wide_pair_clusters(ds->smem_optin) > 0;
+    ds->pairs = false;  // opt-in: nest_datastore_use_cta_pairs
     if (host_status != 0) {
         nest_datastore_destroy(ds);
         return static_cast<nest_status_t>(host_status);
@@ -729,6 +737,14 @@ nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_B, int32_
         }
     }
     return ensure_scratch(ds, need);
+}
+
+nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t on)
+{
+    if (!ds) return NEST_ERR_INVALID_ARG;
+    if (on && !ds->pairs_ok) return NEST_ERR_UNSUPPORTED;
+    ds->pairs = on != 0;
+    return NEST_OK;
 }
 
 nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
@@ -974,7 +990,7 @@ int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r, int32
     SearchPlan sp;
     const nest_status_t st = plan_search(ds, B, r, ragged != 0, &sp);
     if (st != NEST_OK) return -(int32_t)st;
-    return sp.wide ? (sp.wpm.mb == 2 ? 3 : 2) : (sp.tc ? 1 : 0);
+    return sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : 0);
 }
 
 const char* nest_status_string(nest_status_t s)

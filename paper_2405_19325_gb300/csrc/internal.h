@@ -124,6 +124,8 @@ cudaError_t launch_tc_scan(const TcPlan& plan, const CUtensorMap& keys, const CU
 struct WidePlan {
     int nm;       // MMA N = queries per CTA (16, 32, 64, 128 or 256)
     int mb;       // 128-key tiles per pipeline stage (2 only for nm = 256)
+    bool pair;    // nm = 256 on CTA pairs (tcgen05 cta_group::2): 256 keys per tile,
+                  // each part is a pair of CTAs
     int stages;
     int groups;   // query groups of nm
     int parts;    // key-range parts (whole 128-key tiles)
@@ -166,7 +168,11 @@ struct GselectArgs {
     int32_t stage_words;  // shared-memory words per CTA (set by launch_gselect)
 };
 
-bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* plan);
+// Plan of the wide kernel for groups of nm queries; CTA pairs only when `pairs`.
+bool wide_plan_smem(int nm, size_t smem_limit, bool pairs, WidePlan* plan);
+// 2-CTA clusters of the pair kernel the device can hold at once (0: none or
+// the query failed), for the given shared-memory limit per block.
+int wide_pair_clusters(size_t smem_limit);
 // ||q||^2 of B bf16 rows of d elements into qn (fp32, one warp per row).
 cudaError_t launch_wide_qnorm(const void* q, int32_t B, int32_t d, float* qn, cudaStream_t stream);
 cudaError_t launch_tc_wide(const WidePlan& plan, const CUtensorMap& keys,

@@ -12,8 +12,10 @@
 //   2. The main pass streams every key tile once per group of up to 256
 //      queries with tcgen05.mma (M = 128 keys, N = up to 256 queries,
 //      K = 16): tc_wide_kernel keeps one key tile per stage and two TMEM
-//      accumulators of N columns; tc_wide2_kernel (groups of 256) keeps two
-//      key tiles per stage, one accumulator each.  The epilogue warps form
+//      accumulators of N columns.  Groups of 256 run on tc_wide2_kernel
+//      (two key tiles per stage, one accumulator each) or, when asked for,
+//      on CTA pairs (tc_wide_pair_kernel: M = 256 keys over the pair, two
+//      accumulators).  The epilogue warps form
 //      ||q||^2 + ||k||^2 - 2 q.k, admit the keys under each query's threshold
 //      and append them to that query's global list through per-warp slot
 //      reservations.
@@ -267,27 +269,33 @@ __device__ __forceinline__ void wide_release(const int2* resv, int c_begin, int 
 
 // Drains NCOL columns (queries c_base ..) of one TMEM lane (this thread's
 // key row) of an accumulator, starting at tbase, 32 columns per load, and
-// arrives on `release` once they have been read.  With PIPE the next load is
-// in flight while the current columns are tested (more registers); without
-// it the other warps of the SM sub-partition hide the load latency.
-template <int NM, int NCOL, bool PIPE>
+// hands the accumulator back once they have been read: an arrival on
+// `release` in this CTA or, with CLUSTER_RELEASE (a CTA pair), on the even
+// CTA's barrier at the shared::cluster address `release_cluster`.  With PIPE
+// the next load is in flight while the current columns are tested (more
+// registers); without it the other warps of the SM sub-partition hide the
+// load latency.
+template <int NM, int NCOL, bool PIPE, bool CLUSTER_RELEASE = false>
 __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint64_t* release,
                                                int nqv, float kn, bool valid, uint32_t key_idx,
                                                int64_t pos, int lane, const WideShared<NM>& sh,
                                                int2* resv,
-                                               uint32_t* stage, const WideArgs& a, int q0)
+                                               uint32_t* stage, const WideArgs& a, int q0,
+                                               uint32_t release_cluster = 0)
 {
     static_assert(NCOL % 64 == 0 || NCOL == 32, "columns are drained in pairs of 32");
+    auto hand_back = [&] {
+        tc_fence_before();
+        if constexpr (CLUSTER_RELEASE) mbar_arrive_cluster(release_cluster);
+        else mbar_arrive(release);
+    };
     if constexpr (!PIPE) {
 #pragma unroll 1
         for (int c0 = 0; c0 < NCOL; c0 += 32) {
             uint32_t acc[32];
             tmem_ld_32_async(tbase + (uint32_t)c0, acc);
             tmem_wait_ld(acc);
-            if (c0 + 32 == NCOL) {
-                tc_fence_before();
-                mbar_arrive(release);
-            }
+            if (c0 + 32 == NCOL) hand_back();
             wide_columns<32, NM>(acc, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage,
                                  a, q0);
         }
@@ -301,8 +309,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
         if (c0 + 32 < NCOL) {
             tmem_ld_32_async(tbase + (uint32_t)(c0 + 32), a1);
         } else {
-            tc_fence_before();
-            mbar_arrive(release);
+            hand_back();
         }
         wide_columns<32, NM>(a0, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage, a,
                              q0);
@@ -311,8 +318,7 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
             if (c0 + 64 < NCOL) {
                 tmem_ld_32_async(tbase + (uint32_t)(c0 + 64), a0);
             } else {
-                tc_fence_before();
-                mbar_arrive(release);
+                hand_back();
             }
             wide_columns<32, NM>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, pos, lane, sh, resv,
                                  stage, a, q0);
@@ -683,6 +689,202 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
     }
 }
 
+// Groups of 256 queries on CTA pairs (a cluster of two CTAs on one TPC):
+// tcgen05.mma.cta_group::2 with M = 256 keys (128 in each CTA's shared
+// memory and TMEM lanes), N = 256 queries (each CTA stages 128 of them; the
+// MMA reads both halves) and K = 16.  A stage is 16 KiB of keys and 16 KiB
+// of queries per CTA, and TMEM holds two 256-column accumulators, so the
+// epilogue of one 256-key tile overlaps the MMAs of the next (the two-tile
+// kernel above cannot double-buffer: its two tiles fill TMEM).
+//   * both CTAs' TMA loads complete on the even CTA's full barrier, which the
+//     even CTA arms with the pair's bytes; the even CTA's MMA thread issues
+//     for the pair and its commits arrive on both CTAs' empty and acc_full
+//     barriers;
+//   * both CTAs' epilogue threads hand the accumulators back on the even
+//     CTA's acc_empty barrier;
+//   * neither CTA leaves before the other (cluster barrier); a CTA whose wait
+//     gave up pauses first, so that copies in flight land.
+// Key tiles are loaded without an L2 eviction hint: the pairs of different
+// query groups do not keep a fixed order over the same keys, so marking the
+// last group's loads evict-first let lines leave L2 before the other group
+// read them.
+constexpr int kPairStageBytes = 2 * kABytes;  // 128 x 64 keys + 128 x 64 queries
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
+    tc_wide_pair_kernel(const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmQ, const WideArgs a)
+{
+    constexpr int NM = 256;
+    constexpr uint32_t kCols = 512;
+    constexpr int kPairKeys = 2 * kTileM;
+
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    unsigned char* stages = smem;
+    WideShared<NM>& sh =
+        *reinterpret_cast<WideShared<NM>*>(smem + (size_t)a.stages * kPairStageBytes);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t rank = cluster_ctarank();
+    const int cid = blockIdx.x >> 1;  // the pair
+    const int part = cid / a.groups, group = cid - part * a.groups;
+    const int q0 = group * NM;
+    const int nqv = min(NM, a.B - q0);
+
+    const int64_t tiles = (a.N + kPairKeys - 1) / kPairKeys;
+    const int64_t t0 = tiles * part / a.parts, t1 = tiles * (part + 1) / a.parts;
+    const int64_t lo = t0 * kPairKeys;
+    const int64_t hi = min(a.N, t1 * kPairKeys);
+    const int ntiles = (int)(t1 - t0);
+    const int kc = a.kchunks;
+    const int nsteps = ntiles * kc;
+
+    if (tid == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&sh.full[s], 1);
+            mbar_init(&sh.empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&sh.acc_full[b], 1);
+            mbar_init(&sh.acc_empty[b], 2 * kEpiThreads);  // both CTAs' epilogue threads
+        }
+        mbar_init(&sh.drain, 1);
+        sh.abort = 0;
+        sh.issued = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) tmem_alloc_pair(&sh.tmem_base, kCols);
+    tc_fence_before();
+    __syncthreads();
+    // both CTAs' barriers exist before either signals the other's
+    cluster_sync_all();
+    tc_fence_after();
+    const uint32_t tmem = sh.tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer (both CTAs)
+        if (lane == 0 && nsteps > 0) {
+            const uint32_t full_base = mapa_shared(&sh.full[0], 0);
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int s = 0; s < nsteps; ++s) {
+                const int t = s / kc, c = s - t * kc;
+                if (s >= a.stages) {
+                    wait_or_abort_w(&sh.empty[slot], phase ^ 1u, &sh.abort, a.status);
+                    if (*reinterpret_cast<volatile int*>(&sh.abort)) break;
+                }
+                unsigned char* st = stages + (size_t)slot * kPairStageBytes;
+                const uint32_t full0 = full_base + (uint32_t)(slot * sizeof(uint64_t));
+                if (rank == 0) mbar_arrive_expect_tx(&sh.full[slot], 2 * kPairStageBytes);
+                const int32_t y = (int32_t)(lo + (int64_t)t * kPairKeys + kTileM * (int)rank);
+                tma_load_2d_pair(st, &tmK, c * kChunkK, y, full0);
+                tma_load_2d_pair(st + kABytes, &tmQ, c * kChunkK, q0 + kTileM * (int)rank, full0);
+                *reinterpret_cast<volatile int*>(&sh.issued) = s + 1;
+                if (++slot == a.stages) {
+                    slot = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer (even CTA)
+        if (rank == 0 && lane == 0 && nsteps > 0) {
+            constexpr uint32_t idesc = mma_idesc_bf16(2 * kTileM, NM);
+            int slot = 0;
+            uint32_t phase = 0;
+            for (int j = 0; j < ntiles; ++j) {
+                const int buf = j & 1;
+                if (j >= 2)
+                    wait_or_abort_w(&sh.acc_empty[buf], (uint32_t)((j >> 1) - 1) & 1u, &sh.abort,
+                                    a.status);
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * NM);
+                for (int c = 0; c < kc; ++c) {
+                    wait_or_abort_w(&sh.full[slot], phase, &sh.abort, a.status);
+                    tc_fence_after();
+                    const unsigned char* st = stages + (size_t)slot * kPairStageBytes;
+                    const uint64_t ad = smem_desc_sw128(st);
+                    const uint64_t bd = smem_desc_sw128(st + kABytes);
+#pragma unroll
+                    for (int k = 0; k < kChunkK / 16; ++k)
+                        mma_bf16_pair(d_tmem, ad + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
+                    mma_commit_pair_both(&sh.empty[slot]);
+                    if (++slot == a.stages) {
+                        slot = 0;
+                        phase ^= 1u;
+                    }
+                }
+                mma_commit_pair_both(&sh.acc_full[buf]);
+            }
+            // every MMA above has completed once this arrives
+            mma_commit_pair_local(&sh.drain);
+            (void)mbar_wait_bounded(&sh.drain, 0);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue (both CTAs)
+        const int e = tid - 64;
+        const int quarter = warp & 3;
+        for (int j = e; j < NM; j += kEpiThreads) {
+            // padding columns: -1 (never admitted); no sample threshold: every key
+            uint32_t thr = 0xFFFFFFFFu;
+            if (j < nqv) {
+                thr = 0x7FFFFFFFu;
+                if (a.s_sample != nullptr) {
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
+                }
+            }
+            sh.thr[j] = thr;
+            // the pass that admits every key fills whole lists (positions = rows)
+            if (a.s_sample == nullptr && part == 0 && rank == 0 && j < nqv)
+                a.cnt[q0 + j] = (int32_t)a.N;
+            sh.qn[j] = j < nqv ? a.qn[q0 + j] : 0.f;
+        }
+        named_barrier(2, kEpiThreads);
+        int2* resv = sh.resv + (warp - 2) * NM;
+        uint32_t* stage = &sh.stage[warp - 2][0][0];
+        wide_reserve(resv, 0, NM, nqv, lane, a, q0);
+
+        const int64_t ks = a.key_stride;
+        const int row_off = kTileM * (int)rank + 32 * quarter + lane;  // row within a 256-key tile
+        float kn_next = (ntiles > 0 && lo + row_off < hi) ? __ldg(a.knorm + (lo + row_off) * ks) : 0.f;
+        for (int j = 0; j < ntiles; ++j) {
+            const int buf = j & 1;
+            const int64_t row = lo + (int64_t)j * kPairKeys + row_off;
+            const float kn = kn_next;
+            kn_next = (row + kPairKeys < hi) ? __ldg(a.knorm + (row + kPairKeys) * ks) : 0.f;
+            const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
+            const int64_t pos = row < hi ? row : -1;
+            wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
+            tc_fence_after();
+            const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);
+            wide_drain_row<NM, NM, true, true>(tbase, 0, nullptr, nqv, kn, valid,
+                                               (uint32_t)(row * ks), pos, lane, sh, resv, stage, a,
+                                               q0, mapa_shared(&sh.acc_empty[buf], 0));
+        }
+        wide_release(resv, 0, NM, nqv, lane, a, q0);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (*reinterpret_cast<volatile int*>(&sh.abort)) {
+        // a wait gave up: let this CTA's copies in flight land before leaving
+        if (tid == 0) {
+            const uint64_t t_0 = global_timer_ns();
+            while (global_timer_ns() - t_0 < 10000000ull) {
+            }
+        }
+        __syncthreads();
+    }
+    cluster_sync_all();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, kCols);
+    }
+}
+
 // ---------------------------------------------------------------- query norms
 // ||q||^2 of each bf16 query row, one warp per row: lane l sums the squares
 // of 16-byte chunks l, l + 32, ... in order, then the warp adds the lanes'
@@ -912,9 +1114,21 @@ size_t wide_fixed()
 }
 
 template <int NM>
-bool wide_plan_nm(size_t smem_limit, WidePlan* p)
+bool wide_plan_nm(size_t smem_limit, bool pairs, WidePlan* p)
 {
     const size_t fixed = wide_fixed<NM>();
+    p->pair = false;
+    if (NM == 256 && pairs && fixed + 4 * (size_t)kPairStageBytes <= smem_limit) {
+        // CTA pairs: 32 KiB stages per CTA, double-buffered accumulators
+        int stages = (int)((smem_limit - fixed) / kPairStageBytes);
+        stages = stages > kMaxStagesW ? kMaxStagesW : stages;
+        p->nm = NM;
+        p->mb = 2;
+        p->pair = true;
+        p->stages = stages;
+        p->smem = fixed + (size_t)stages * kPairStageBytes;
+        return true;
+    }
     if (NM == 256) {
         // two key tiles per stage when three 64 KiB stages fit
         const size_t st2 = (size_t)(2 * kABytes + NM * kChunkK * 2);
@@ -943,6 +1157,13 @@ template <int NM>
 cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
                            const WideArgs& a, cudaStream_t stream)
 {
+    if (NM == 256 && p.pair) {
+        cudaError_t e =
+            raise_smem_limit(reinterpret_cast<const void*>(tc_wide_pair_kernel), (int)p.smem);
+        if (e != cudaSuccess) return e;
+        tc_wide_pair_kernel<<<2 * p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
+        return cudaGetLastError();
+    }
     if (NM == 256 && p.mb == 2) {
         cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_wide2_kernel), (int)p.smem);
         if (e != cudaSuccess) return e;
@@ -959,16 +1180,38 @@ cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUte
 
 }  // namespace
 
-bool wide_plan_smem(int nm, size_t smem_limit, WidePlan* p)
+bool wide_plan_smem(int nm, size_t smem_limit, bool pairs, WidePlan* p)
 {
     switch (nm) {
-    case 16: return wide_plan_nm<16>(smem_limit, p);
-    case 32: return wide_plan_nm<32>(smem_limit, p);
-    case 64: return wide_plan_nm<64>(smem_limit, p);
-    case 128: return wide_plan_nm<128>(smem_limit, p);
-    case 256: return wide_plan_nm<256>(smem_limit, p);
+    case 16: return wide_plan_nm<16>(smem_limit, pairs, p);
+    case 32: return wide_plan_nm<32>(smem_limit, pairs, p);
+    case 64: return wide_plan_nm<64>(smem_limit, pairs, p);
+    case 128: return wide_plan_nm<128>(smem_limit, pairs, p);
+    case 256: return wide_plan_nm<256>(smem_limit, pairs, p);
     default: return false;
     }
+}
+
+int wide_pair_clusters(size_t smem_limit)
+{
+    WidePlan p{};
+    if (!wide_plan_nm<256>(smem_limit, true, &p) || !p.pair) return 0;
+    if (raise_smem_limit(reinterpret_cast<const void*>(tc_wide_pair_kernel), (int)p.smem) !=
+        cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2, 1, 1);
+    cfg.blockDim = dim3(kTcThreads, 1, 1);
+    cfg.dynamicSmemBytes = p.smem;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(tc_wide_pair_kernel),
+                                       &cfg) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return 0;
+    }
+    return n;
 }
 
 cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,

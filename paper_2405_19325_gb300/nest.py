@@ -33,6 +33,7 @@ SIGNATURES = {
                                              ctypes.POINTER(_P)]),
     "nest_datastore_destroy": (ctypes.c_int, [_P]),
     "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
+    "nest_datastore_use_cta_pairs": (ctypes.c_int, [_P, _I32]),
     "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_static": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_masked": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P, _P]),
@@ -159,6 +160,12 @@ class Datastore:
     def reserve(self, max_B: int, max_r: int, ragged: bool = False) -> None:
         _check(self._lib.nest_datastore_reserve(self._h, max_B, max_r, int(ragged)),
                "nest_datastore_reserve")
+
+    def use_cta_pairs(self, on: bool) -> None:
+        """Groups of 256 queries on CTA pairs (opt-in) or on single CTAs with
+        two key tiles per stage (default)."""
+        _check(self._lib.nest_datastore_use_cta_pairs(self._h, int(bool(on))),
+               "nest_datastore_use_cta_pairs")
 
     # ------------------------------------------------------------ search / mix / step
     def search(self, q: torch.Tensor, r: int, seg_off: torch.Tensor | None = None,
@@ -355,7 +362,7 @@ class Datastore:
         return int(self._lib.nest_launch_count(self._h))
 
     SEARCH_PATHS = {0: "scan_topr_kernel", 1: "tc_scan_kernel", 2: "tc_wide_kernel",
-                    3: "tc_wide2_kernel"}
+                    3: "tc_wide2_kernel", 4: "tc_wide_pair_kernel"}
 
     def search_path(self, B: int, r: int, ragged: bool = False) -> str:
         """Name of the distance-scan kernel a search of this shape runs."""

@@ -101,12 +101,17 @@ def test_verify_spans_matches_oracle(nest):
 @pytest.mark.parametrize("path,B,r,dtype,N", [("tc_scan_kernel", 4, 64, "bf16", 60000),
                                                ("tc_wide_kernel", 40, 128, "bf16", 60000),
                                                ("scan_topr_kernel", 3, 50, "f32", 60000),
-                                               # groups of 256: one pass, then two passes
+                                               # groups of 256: one pass, then two passes,
+                                               # on CTA pairs and on single CTAs
+                                               ("tc_wide_pair_kernel", 300, 128, "bf16", 60000),
+                                               ("tc_wide_pair_kernel", 260, 64, "bf16", 140000),
                                                ("tc_wide2_kernel", 300, 128, "bf16", 60000),
                                                ("tc_wide2_kernel", 260, 64, "bf16", 140000)])
 def test_masked_search_skips_used_keys(nest, path, B, r, dtype, N):
     K, V, q, p_lm = _case(N, 256, B, 300, seed=42, dtype=dtype)
     ds = nest.Datastore(K, V, 300)
+    if path == "tc_wide_pair_kernel":
+        ds.use_cta_pairs(True)
     assert ds.search_path(B, r) == path
     mask = ds.new_key_mask()
     g = torch.Generator().manual_seed(43)

@@ -38,16 +38,19 @@ def _cand_counts(B, N, seg_off):
 
 
 def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, exact=False,
-                  oracle_threads=None, check_rows=None):
+                  oracle_threads=None, check_rows=None, pairs=None):
     """GPU step through the C ABI, then the oracle on the same bytes.
 
     ``check_rows`` restricts the oracle (and the comparison) to those query
     rows of a full-scan batch; the GPU always runs the whole batch.
+    ``pairs`` chooses CTA pairs or single CTAs for groups of 256 queries.
     """
     dev = torch.device("cuda")
     K, V, q, p_lm = K.to(dev), V.to(dev), q.to(dev), p_lm.to(dev)
     so = seg_off.to(dev) if seg_off is not None else None
     ds = nest.Datastore(K, V, vocab)
+    if pairs is not None:
+        ds.use_cta_pairs(pairs)
     out = ds.step(q, r, p_lm, mu, lam, seg_off=so, want_p_knn=True)
     torch.cuda.synchronize()
     assert ds.device_status() == 0
@@ -342,21 +345,29 @@ def test_wide_batch_single_pass_over_300_queries(nest):
     run_and_check(nest, K, V, q, p_lm, 64, 1 / np.sqrt(128), 0.8, 500, "bf16")
 
 
+def _group256_path(pairs):
+    return "tc_wide_pair_kernel" if pairs else "tc_wide2_kernel"
+
+
+@pytest.mark.parametrize("pairs", [True, False], ids=["cta_pairs", "two_tiles"])
 @pytest.mark.parametrize("N,d,B,r", [
-    (200036, 200, 260, 64),   # two passes; last pair: one partial tile, one tile past N
+    (200036, 200, 260, 64),   # two passes; last 256-key tile: part real, part past N
     (70017, 64, 256, 33),     # single pass, one full group, d = one K chunk, 1-row tile
 ])
-def test_two_tile_wide_kernel_edges(nest, N, d, B, r):
-    """Groups of 256 queries run two 128-key tiles per pipeline stage: a
+def test_group256_wide_kernel_edges(nest, N, d, B, r, pairs):
+    """Groups of 256 queries, on CTA pairs (256-key tiles split over two
+    SMs) and on single CTAs (two 128-key tiles per pipeline stage): a
     partial last group (padding columns), d not a multiple of 64 (the last
-    K chunk half outside the rows), and a last tile pair whose second tile
-    lies wholly past the last key."""
+    K chunk half outside the rows), and a last 256-key tile whose second
+    half lies wholly past the last key."""
     K, V, q, p_lm = _random_case(N, d, B, 900, "bf16", seed=23 + d, centres=48)
     ds = nest.Datastore(K.cuda(), V.cuda(), 900)
-    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.use_cta_pairs(pairs)
+    assert ds.search_path(B, r) == _group256_path(pairs)
     ds.close()
     rows = list(range(0, B, 7)) + [B - 1]
-    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 900, "bf16", check_rows=rows)
+    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 900, "bf16", check_rows=rows,
+                  pairs=pairs)
 
 
 @pytest.mark.parametrize("N,r,masked", [
@@ -395,7 +406,8 @@ def test_wide_batch_list_lengths_that_split_a_warp(nest, N, r, masked):
     ds.close()
 
 
-def test_wide_batch_keys_stored_cluster_by_cluster(nest):
+@pytest.mark.parametrize("pairs", [True, False], ids=["cta_pairs", "two_tiles"])
+def test_wide_batch_keys_stored_cluster_by_cluster(nest, pairs):
     """Keys stored cluster after cluster (as a datastore built document by
     document would be): each query's main-pass survivors come from the one or
     two key ranges that hold its cluster, so the epilogue warps there use up
@@ -411,13 +423,16 @@ def test_wide_batch_keys_stored_cluster_by_cluster(nest):
     V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
     p_lm = torch.softmax(torch.randn(B, vocab, generator=g) * 2, dim=1)
     ds = nest.Datastore(K.cuda(), V.cuda(), vocab)
-    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.use_cta_pairs(pairs)
+    assert ds.search_path(B, r) == _group256_path(pairs)
     ds.close()
     rows = list(range(0, B, 37)) + [B - 1]
-    run_and_check(nest, K, V, q, p_lm, r, 1 / 16, 0.8, vocab, "bf16", check_rows=rows)
+    run_and_check(nest, K, V, q, p_lm, r, 1 / 16, 0.8, vocab, "bf16", check_rows=rows,
+                  pairs=pairs)
 
 
-def test_wide_batch_massive_exact_ties(nest):
+@pytest.mark.parametrize("pairs", [True, False], ids=["cta_pairs", "two_tiles"])
+def test_wide_batch_massive_exact_ties(nest, pairs):
     """Groups of 256 queries over keys that are exact copies of two integer
     vectors (two of every three keys are the same vector): every query sees
     two distances, the r nearest are the r smallest indices among the nearer
@@ -435,10 +450,12 @@ def test_wide_batch_massive_exact_ties(nest):
     V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
     p_lm = torch.softmax(torch.randn(B, vocab, generator=g), dim=1)
     ds = nest.Datastore(K.cuda(), V.cuda(), vocab)
-    assert ds.search_path(B, r) == "tc_wide2_kernel"
+    ds.use_cta_pairs(pairs)
+    assert ds.search_path(B, r) == _group256_path(pairs)
     ds.close()
     rows = list(range(0, B, 23)) + [B - 1]
-    run_and_check(nest, K, V, q, p_lm, r, 1 / 8, 0.7, vocab, "bf16", exact=True, check_rows=rows)
+    run_and_check(nest, K, V, q, p_lm, r, 1 / 8, 0.7, vocab, "bf16", exact=True, check_rows=rows,
+                  pairs=pairs)
 
 
 def test_large_batch_shape_sampled_rows(nest):

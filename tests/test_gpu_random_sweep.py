@@ -15,7 +15,8 @@ branch on (tile and warp multiples, the 8,192-word copy stride of the
 selection, the 65,536-key threshold sample, the query-group sizes, list
 lengths around 1,024) and goes through each public entry point in turn:
 the device step, the host-buffer step, search + Eq. 4 + the Eq. 5 / Eq. 6
-decision, and the masked search.
+decision, and the masked search.  In both sets, half of the bf16 shapes (by
+seed) run groups of 256 queries on CTA pairs.
 """
 import numpy as np
 import pytest
@@ -97,11 +98,17 @@ def _draw_edge_cases():
 EDGE_CASES = _draw_edge_cases()
 
 
+def _pairs(c):
+    """Half of the bf16 shapes (by seed) run groups of 256 queries on CTA pairs."""
+    return c["dtype"] == "bf16" and c["seed"] % 2 == 1
+
+
 def _case_id(c):
     entry = c.get("entry")
     return (f"{c['dtype']}-N{c['N']}-d{c['d']}-B{c['B']}-r{c['r']}-{c['layout']}"
             + ("-ragged" if c["ragged"] else "")
-            + (f"-{entry}" if entry else ("-masked" if c["masked"] else "")))
+            + (f"-{entry}" if entry else ("-masked" if c["masked"] else ""))
+            + ("-pairs" if _pairs(c) else ""))
 
 
 @pytest.fixture(scope="module")
@@ -178,6 +185,8 @@ def _run_case(nest, c):
     K, V, q, p_lm, seg_off, excl = _inputs(c, vocab)
     dev = torch.device("cuda")
     ds = nest.Datastore(K.to(dev), V.to(dev), vocab)
+    if _pairs(c):
+        ds.use_cta_pairs(True)
     qd = q.to(dev)
     so_d = seg_off.to(dev) if seg_off is not None else None
     mu, lam = 1 / np.sqrt(d), 0.75
@@ -253,9 +262,12 @@ def test_sweep_reaches_every_search_path(nest):
     for c in CASES + EDGE_CASES:
         K = torch.zeros(64, c["d"], dtype=synth.torch_dtype(c["dtype"]), device="cuda")
         ds = nest.Datastore(K, V, 10)
+        if _pairs(c):
+            ds.use_cta_pairs(True)
         seen.add(ds.search_path(c["B"], c["r"], ragged=c["ragged"]))
         ds.close()
-    assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel", "scan_topr_kernel"}, seen
+    assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
+                    "tc_wide_pair_kernel", "scan_topr_kernel"}, seen
 
 
 # ---------------------------------------------------------------- Eq. 7 verification and masking
