@@ -315,17 +315,6 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const void* tmap, in
         : "memory");
 }
 
-__device__ __forceinline__ void tma_load_2d_pair_hint(void* dst, const void* tmap, int32_t x,
-                                                      int32_t y, uint32_t bar_cluster,
-                                                      uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(dst)),
-        "l"(tmap), "r"(x), "r"(y), "r"(bar_cluster), "l"(policy)
-        : "memory");
-}
-
 // TMEM columns shared by the pair: one warp of each CTA calls these, and
 // both get the same address.
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst_smem, uint32_t ncols)
