@@ -454,6 +454,27 @@ def measure(args, w, x_all, ds, B, world, rank, local):
                     "tensor_frac": alg_flops / (scan_avg_ms / 1e3) / 1e12 / tc_peak,
                     "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
 
+    # ---- the search alone (scan and merge or selection, no mix), same batch
+    s_buf = torch.empty(B, w.r, dtype=torch.float32, device=x.q.device)
+    i_buf = torch.empty(B, w.r, dtype=torch.int64, device=x.q.device)
+    n_search = max(1, min(args.steps, 200))
+    for _ in range(3):
+        ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
+    barrier(world)
+    torch.cuda.synchronize()
+    u0 = torch.cuda.Event(enable_timing=True)
+    u1 = torch.cuda.Event(enable_timing=True)
+    u0.record(stream)
+    for _ in range(n_search):
+        ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
+    u1.record(stream)
+    torch.cuda.synchronize()
+    search_ms = max_over_ranks(u0.elapsed_time(u1), world) / n_search
+    if ds.device_status() != 0:
+        raise SystemExit("device status error during the search-only steps")
+    search = {"call": "nest_knn_search", "ms": search_ms,
+              "queries_per_s": world * B / (search_ms / 1e3), "steps": n_search}
+
     # ---- end to end through the public API with pinned host buffers
     q_h = x.q.cpu().pin_memory()
     p_h = x.p_lm.cpu().pin_memory()
@@ -504,7 +525,7 @@ def measure(args, w, x_all, ds, B, world, rank, local):
             "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
             "data": "synthetic", "config": config_of(w, x, args.pipeline),
             "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "search": search,
             "gpu_launches": launches, "clocks": clk,
         }
     return line
