@@ -23,6 +23,7 @@ import argparse
 import json
 import os
 import statistics
+import platform
 import subprocess
 import sys
 import time
@@ -232,6 +233,10 @@ class OracleSampler:
             return self.nq / seconds
         return self.nq * (n / self.N) / seconds
 
+    def keys_per_s(self, n: int, seconds: float) -> float:
+        """(query, key) distance evaluations per second of the sample."""
+        return (self.n if self.ragged else self.nq * n) / seconds
+
     def describe(self, n: int) -> str:
         w = self.w
         if self.ragged:
@@ -242,13 +247,29 @@ class OracleSampler:
                 f"linear in the keys scanned)")
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (or architecture) from /proc/cpuinfo."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            text = f.read()
+    except OSError:
+        return platform.machine()
+    for key in ("model name", "Model Name", "CPU part"):
+        for line in text.splitlines():
+            if line.split(":")[0].strip() == key:
+                val = line.split(":", 1)[1].strip()
+                return val if key != "CPU part" else f"{platform.machine()} (CPU part {val})"
+    return platform.machine()
+
+
 def cpu_baseline(w, x, nq: int, budget_s: float = 15.0):
     """The oracle on the host cores: one bounded sample of ~budget_s seconds."""
     smp = OracleSampler(w, x, nq)
     n = smp.fit(budget_s)
     sec = smp.run(n)
     return {"value": smp.queries_per_s(n, sec), "unit": "queries/s", "cores": smp.threads,
-            "kind": "oracle", "sample": smp.describe(n), "seconds": sec}
+            "kind": "oracle", "sample": smp.describe(n), "seconds": sec,
+            "keys_per_s": smp.keys_per_s(n, sec), "cpu": cpu_model()}
 
 
 def run_reference(args, w, world, rank):
@@ -276,7 +297,9 @@ def run_reference(args, w, world, rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_of(w, x),
         "cpu_baseline": {"value": value, "unit": "queries/s", "cores": smp.threads,
-                         "kind": "oracle", "sample": smp.describe(n)},
+                         "kind": "oracle", "sample": smp.describe(n),
+                         "keys_per_s": smp.keys_per_s(n, total / len(times)),
+                         "cpu": cpu_model()},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
