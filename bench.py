@@ -22,8 +22,8 @@ from __future__ import annotations
 import argparse
 import json
 import os
-import statistics
 import platform
+import statistics
 import subprocess
 import sys
 import time
