@@ -405,6 +405,38 @@ def make_step(args, w, x, ds):
                   "lambda_t+relaxed speculative acceptance) of one drafted span")
 
 
+def graph_replay(step, stream, args, world, B):
+    """Times the step replayed from a CUDA graph (captured once, after the
+    warm-up has sized the scratch, so that nothing allocates during capture);
+    this removes the host's launch work and most gaps between kernels."""
+    n = max(1, min(args.steps, 200))
+    try:
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            step()
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            step()
+        for _ in range(3):
+            g.replay()
+        barrier(world)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+    except RuntimeError as err:
+        return {"error": str(err).splitlines()[0][:200]}
+    ms = max_over_ranks(e0.elapsed_time(e1), world) / n
+    return {"ms_per_step": ms, "value": world * B / (ms / 1e3), "steps": n}
+
+
 def measure(args, w, x_all, ds, B, world, rank, local):
     """Time one batch size on an existing datastore; returns the JSON line (rank 0)."""
     x = synth.Inputs(K=x_all.K, V=x_all.V, q=x_all.q[:B].contiguous(),
@@ -476,6 +508,11 @@ def measure(args, w, x_all, ds, B, world, rank, local):
                     "alg_bytes_per_launch": alg_bytes, "alg_flops_per_launch": alg_flops,
                     "tensor_frac": alg_flops / (scan_avg_ms / 1e3) / 1e12 / tc_peak,
                     "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
+
+    # ---- the same step captured once in a CUDA graph and replayed
+    graph = graph_replay(step, stream, args, world, B)
+    if ds.device_status() != 0:
+        raise SystemExit("device status error during the graph replays")
 
     # ---- the search alone (scan and merge or selection, no mix), same batch
     s_buf = torch.empty(B, w.r, dtype=torch.float32, device=x.q.device)
@@ -549,6 +586,7 @@ def measure(args, w, x_all, ds, B, world, rank, local):
             "data": "synthetic", "config": config_of(w, x, args.pipeline),
             "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "search": search,
+            "graph": graph,
             "gpu_launches": launches, "clocks": clk,
         }
     return line
