@@ -324,6 +324,19 @@ NEST_API nest_status_t nest_verify_spans(nest_datastore_t* ds, const float* p_m,
                                          int32_t* n_accept_out, void* stream);
 
 /*
+ * Check of the failure-detection path (no counterpart in the paper).  Runs
+ * one kernel that waits on an mbarrier nothing arrives on, through the same
+ * bounded wait the scan kernels use for their pipeline stages.  The wait
+ * gives up after its limit (2 s) and records NEST_ERR_TIMEOUT in this
+ * datastore's device status, which nest_device_status then returns; the
+ * context stays usable.  Synchronizes `stream`.  waited_ns (host, may be
+ * NULL) receives how long the kernel waited.  Returns NEST_OK when the
+ * kernel ran.
+ */
+NEST_API nest_status_t nest_selftest_bounded_wait(nest_datastore_t* ds, int64_t* waited_ns,
+                                                  void* stream);
+
+/*
  * Synchronize `stream`, return the first condition the GPU recorded for
  * this datastore since the previous call (NEST_OK if none), and clear it.
  */

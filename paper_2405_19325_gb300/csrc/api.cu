@@ -945,6 +945,24 @@ nest_status_t nest_verify_spans(nest_datastore_t* ds, const float* p_m, const in
     return NEST_OK;
 }
 
+nest_status_t nest_selftest_bounded_wait(nest_datastore_t* ds, int64_t* waited_ns, void* stream)
+{
+    if (!ds) return NEST_ERR_INVALID_ARG;
+    cudaStream_t st = as_stream(stream);
+    int64_t* d_ns = nullptr;
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&d_ns), sizeof(int64_t));
+    if (e == cudaSuccess) e = launch_wait_selftest(ds->status, d_ns, st);
+    int64_t h_ns = 0;
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&h_ns, d_ns, sizeof(int64_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (d_ns) (void)cudaFree(d_ns);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
+    if (waited_ns) *waited_ns = h_ns;
+    return NEST_OK;
+}
+
 nest_status_t nest_device_status(nest_datastore_t* ds, void* stream)
 {
     if (!ds) return NEST_ERR_INVALID_ARG;

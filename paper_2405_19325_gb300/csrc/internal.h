@@ -168,6 +168,11 @@ struct GselectArgs {
     int32_t stage_words;  // shared-memory words per CTA (set by launch_gselect)
 };
 
+// ---------------------------------------------------------------- selftest.cu
+// One kernel whose bounded mbarrier wait runs out: records NEST_ERR_TIMEOUT
+// in *status and the nanoseconds it waited in *waited_ns (device memory).
+cudaError_t launch_wait_selftest(int* status, int64_t* waited_ns, cudaStream_t stream);
+
 // Plan of the wide kernel for groups of nm queries; CTA pairs only when `pairs`.
 bool wide_plan_smem(int nm, size_t smem_limit, bool pairs, WidePlan* plan);
 // 2-CTA clusters of the pair kernel the device can hold at once (0: none or

@@ -34,6 +34,7 @@ SIGNATURES = {
     "nest_datastore_destroy": (ctypes.c_int, [_P]),
     "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
     "nest_datastore_use_cta_pairs": (ctypes.c_int, [_P, _I32]),
+    "nest_selftest_bounded_wait": (ctypes.c_int, [_P, ctypes.POINTER(_I64), _P]),
     "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_static": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_masked": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P, _P]),
@@ -341,6 +342,14 @@ class Datastore:
         return {"p_m": st["p_m"], "s": st["s"], "idx": st["idx"]}
 
     # ------------------------------------------------------------ status / timing
+    def selftest_bounded_wait(self, stream=None) -> int:
+        """Runs a kernel whose bounded wait runs out (nothing arrives); the
+        device status then holds NEST_ERR_TIMEOUT.  Returns the nanoseconds
+        the kernel waited."""
+        ns = ctypes.c_int64()
+        _check(self._lib.nest_selftest_bounded_wait(self._h, ctypes.byref(ns), _stream(stream)),
+               "nest_selftest_bounded_wait")
+        return ns.value
     def device_status(self, stream=None) -> int:
         """Synchronize and return (and clear) the device status code."""
         return int(self._lib.nest_device_status(self._h, _stream(stream)))

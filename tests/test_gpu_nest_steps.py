@@ -160,3 +160,25 @@ def test_masked_ragged_search(nest):
     check_search(s.cpu().numpy(), idx.cpu().numpy(), s_or, i_or, K_np, q_np, "bf16", counts)
     assert (idx[3] == -1).all()
     ds.close()
+
+
+def test_bounded_wait_gives_up_and_the_context_stays_usable(nest):
+    """Failure detection without a fault: a kernel waits, through the scan
+    kernels' bounded mbarrier wait, on a barrier nothing arrives on.  It must
+    give up after about 2 s, the device status must read NEST_ERR_TIMEOUT
+    (and be cleared by reading it), and a search afterwards must still run
+    and match the oracle."""
+    K, V, q, p_lm = _case(20000, 256, 4, 300, seed=45)
+    ds = nest.Datastore(K, V, 300)
+    waited = ds.selftest_bounded_wait()
+    assert 1.9e9 <= waited <= 4e9, waited
+    assert ds.device_status() == 8  # NEST_ERR_TIMEOUT
+    assert ds.device_status() == 0
+    s, idx = ds.search(q, 64)
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    K_np, q_np = synth.to_numpy_raw(K), synth.to_numpy_raw(q)
+    s_or, i_or = oracle.knn_search(K_np, q_np, 64)
+    check_search(s.cpu().numpy(), idx.cpu().numpy(), s_or, i_or, K_np, q_np, "bf16",
+                 np.full(4, 20000))
+    ds.close()
