@@ -258,7 +258,11 @@ def cpu_model() -> str:
         for line in text.splitlines():
             if line.split(":")[0].strip() == key:
                 val = line.split(":", 1)[1].strip()
-                return val if key != "CPU part" else f"{platform.machine()} (CPU part {val})"
+                if key != "CPU part":
+                    return val
+                names = {"0xd4f": "Arm Neoverse V2", "0xd40": "Arm Neoverse V1",
+                         "0xd0c": "Arm Neoverse N1", "0xd49": "Arm Neoverse N2"}
+                return f"{platform.machine()} {names.get(val, 'CPU part ' + val)}"
     return platform.machine()
 
 
