@@ -57,6 +57,9 @@ def parse():
                    help="knnlm: search + Eq. 2 + Eq. 3 (default); nest: masked search + Eq. 2 + "
                         "Eq. 4 + Eq. 5/6 decision; verify: a batch of drafted positions "
                         "searched, mixed (Eq. 4) and verified (Eq. 7)")
+    p.add_argument("--cta-pairs", action="store_true",
+                   help="run groups of 256 queries on CTA pairs (nest_datastore_use_cta_pairs) "
+                        "instead of the default two-tile kernel")
     p.add_argument("--sweep", default=None,
                    help="comma-separated query batch sizes measured on one datastore, one JSON "
                         "line each (e.g. 1,8,64,256 for the d=8192 workload)")
@@ -362,6 +365,8 @@ def main():
     B_gen = max(b for b in sweep if b is not None) if any(b is not None for b in sweep) else None
     x = synth.make_inputs(w, device=dev, B=B_gen, N=args.N, seed=w.seed + rank)
     ds = nest.Datastore(x.K, x.V, w.vocab)
+    if args.cta_pairs:
+        ds.use_cta_pairs(True)
     for B in sweep:
         line = measure(args, w, x, ds, B if B is not None else x.q.shape[0], world, rank, local)
         if rank == 0:

@@ -110,8 +110,8 @@ NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_
  * A pair splits each 256-key tile over two SMs and double-buffers its
  * accumulators; with one query group it runs as fast as path 3, but with
  * several groups their pairs drift apart and read the same keys from DRAM
- * again (1.22 times the key bytes at 1M keys and B = 512 on a GB300,
- * against 1.11 for path 3), so path 3 stays the default.  Pairs need two
+ * again (1.20 times the key bytes at 1M keys and B = 512 on a GB300,
+ * against 1.09 for path 3), so path 3 stays the default.  Pairs need two
  * CTAs of about 220 KiB of shared memory each on the two SMs of one TPC at
  * the same time; on = 1 where the device cannot place them returns
  * NEST_ERR_UNSUPPORTED and changes nothing.  Host only; takes effect from
