@@ -313,7 +313,8 @@ NEST_API nest_status_t nest_knn_decide(nest_datastore_t* ds, const float* p_m, c
  *
  * 1 <= rows <= 65535 and 1 <= spans <= 65535; a span may be empty
  * (span_off[j] == span_off[j+1], n_accept = 0).
- * gamma in (0, 1] is the relaxation factor.  A draft token outside
+ * gamma > 0 is the relaxation factor (Sec. 3.4 relaxes with values in
+ * (0, 1]; gamma <= 0 or NaN is refused).  A draft token outside
  * [0, vocab) is rejected and recorded as NEST_ERR_VALUE_RANGE; bad span
  * offsets give n_accept = 0 and NEST_ERR_INVALID_ARG in the device status.
  */
