@@ -19,9 +19,11 @@
  *     by the caller, unless a comment says otherwise.  Matrices are dense and
  *     row-major.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
- *     stream).  All work is stream-ordered and no call synchronizes the
- *     stream, except nest_datastore_create, nest_device_status and
- *     nest_timing_read, which say so.
+ *     stream).  All work is stream-ordered and no call synchronizes, except
+ *     nest_datastore_create, nest_datastore_destroy, nest_knn_step_host,
+ *     nest_device_status, nest_selftest_bounded_wait and nest_timing_read,
+ *     and a call that allocates scratch (nest_datastore_reserve, or the
+ *     first search of a larger shape without it); each says so.
  *   - Keys and queries are NEST_F32 or NEST_BF16 (IEEE bfloat16 bits).
  *     Distances, similarities and probabilities are fp32.
  *   - Argument errors are found on the host before anything is launched and
@@ -374,7 +376,8 @@ NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
 /* Static text for a status code. */
 NEST_API const char* nest_status_string(nest_status_t status);
 
-/* ABI version: major * 10000 + minor * 100 + patch. */
+/* ABI version: major * 10000 + minor * 100 + patch (0.2.0: CTA pairs and
+ * the bounded-wait self-test added to 0.1.0). */
 NEST_API int32_t nest_version(void);
 
 #ifdef __cplusplus

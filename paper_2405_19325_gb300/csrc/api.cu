@@ -1028,7 +1028,7 @@ const char* nest_status_string(nest_status_t s)
     return "unknown status";
 }
 
-int32_t nest_version(void) { return 100; }
+int32_t nest_version(void) { return 200; }
 
 }  // extern "C"
 
