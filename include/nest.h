@@ -370,6 +370,37 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,
                                   int32_t ragged);
 
+/*
+ * The plan a search of this shape would run, computed on the host without
+ * a GPU or a handle (no counterpart in the paper; for capacity planning and
+ * for tests of the planning logic).  It runs the same planning code as
+ * nest_knn_search on a datastore of N keys of d elements of `dtype`, on a
+ * device with `num_sms` SMs and `smem_per_block` bytes of opt-in shared
+ * memory per block (cudaDevAttrMaxSharedMemoryPerBlockOptin), with
+ * nest_datastore_use_cta_pairs(ds, cta_pairs) in effect (the device is
+ * assumed able to place the pairs).  Arguments are checked as
+ * nest_datastore_create and nest_knn_search check them.
+ */
+typedef struct nest_plan {
+    int32_t path;               /* as nest_search_path */
+    int32_t queries_per_group;  /* queries one CTA (or CTA pair) scans together */
+    int32_t groups;             /* query groups */
+    int32_t parts;              /* key-range parts per group (CTAs or CTA pairs) */
+    int32_t stages;             /* pipeline stages of the scan kernel */
+    int32_t single_pass;        /* paths 2-4: 1 when the sample is every key */
+    int64_t sample_stride;      /* paths 2-4: the sample is every stride-th key */
+    int64_t list_capacity;      /* words of a query's candidate list: in a CTA's shared
+                                   memory (paths 0-1), or in global memory for the
+                                   thresholded pass, or the whole datastore when
+                                   single_pass (2-4) */
+    int64_t scratch_bytes;      /* scratch the handle allocates for this search */
+} nest_plan_t;
+
+NEST_API nest_status_t nest_plan_offline(int64_t N, int32_t d, nest_dtype_t dtype, int32_t B,
+                                         int32_t r, int32_t ragged, int32_t num_sms,
+                                         int64_t smem_per_block, int32_t cta_pairs,
+                                         nest_plan_t* out);
+
 /* Kernels this handle has launched since it was created (all kinds). */
 NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
 

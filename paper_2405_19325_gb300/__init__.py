@@ -3,6 +3,6 @@
 The path (search, Eq. 2, Eq. 3 / Eq. 4) runs in hand-written CUDA kernels
 behind the C ABI of include/nest.h; ``nest.Datastore`` is the Python binding.
 """
-from .nest import BF16, F32, LIB_PATH, Datastore, NestError, load_library  # noqa: F401
+from .nest import BF16, F32, LIB_PATH, Datastore, NestError, load_library, plan_offline  # noqa: F401
 
-__all__ = ["Datastore", "NestError", "load_library", "LIB_PATH", "F32", "BF16"]
+__all__ = ["Datastore", "NestError", "load_library", "plan_offline", "LIB_PATH", "F32", "BF16"]

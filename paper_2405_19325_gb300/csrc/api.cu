@@ -1002,6 +1002,54 @@ nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, int64_t* 
 
 int64_t nest_launch_count(const nest_datastore_t* ds) { return ds ? ds->launches : 0; }
 
+nest_status_t nest_plan_offline(int64_t N, int32_t d, nest_dtype_t dtype, int32_t B, int32_t r,
+                                int32_t ragged, int32_t num_sms, int64_t smem_per_block,
+                                int32_t cta_pairs, nest_plan_t* out)
+{
+    if (!out) return NEST_ERR_INVALID_ARG;
+    if (dtype != NEST_F32 && dtype != NEST_BF16) return NEST_ERR_DTYPE;
+    if (N < 1 || N > kMaxKeys || d < 1 || B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R ||
+        num_sms < 2 || smem_per_block < 1)
+        return NEST_ERR_INVALID_ARG;
+    const int64_t row_bytes = (int64_t)d * element_size(dtype);
+    if (row_bytes > NEST_MAX_ROW_BYTES) return NEST_ERR_UNSUPPORTED;
+    if (row_bytes % 16 != 0) return NEST_ERR_ALIGN;
+    nest_datastore ds;
+    ds.N = N;
+    ds.d = d;
+    ds.dtype = dtype;
+    ds.row_bytes = (int32_t)row_bytes;
+    ds.num_sms = num_sms;
+    ds.smem_optin = (size_t)smem_per_block;
+    // the key tensor map encodes for every such bf16 datastore (16-byte rows)
+    ds.tc = dtype == NEST_BF16 && N <= (int64_t)0x7FFFFF00;
+    ds.pairs_ok = ds.tc;
+    ds.pairs = ds.tc && cta_pairs != 0;
+    SearchPlan sp;
+    const nest_status_t st = plan_search(&ds, B, r, ragged != 0, &sp);
+    if (st != NEST_OK) return st;
+    nest_plan_t p{};
+    p.path = sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : 0);
+    if (sp.wide) {
+        p.queries_per_group = sp.wpm.nm;
+        p.groups = sp.wpm.groups;
+        p.parts = sp.wpm.parts;
+        p.stages = sp.wpm.stages;
+        p.single_pass = sp.single_pass ? 1 : 0;
+        p.sample_stride = sp.stride;
+        p.list_capacity = sp.single_pass ? sp.cap_s : sp.cap_m;
+    } else {
+        p.queries_per_group = sp.nq;
+        p.groups = sp.groups;
+        p.parts = sp.parts;
+        p.stages = sp.tc ? sp.tcp.stages : sp.scan.stages;
+        p.list_capacity = sp.tc ? sp.tcp.cap : sp.scan.cap;
+    }
+    p.scratch_bytes = (int64_t)(sp.total_words * sizeof(uint64_t));
+    *out = p;
+    return NEST_OK;
+}
+
 int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r, int32_t ragged)
 {
     if (!ds || B < 1 || B > kMaxB || r < 1 || r > NEST_MAX_R) return -(int32_t)NEST_ERR_INVALID_ARG;

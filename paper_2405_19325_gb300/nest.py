@@ -35,6 +35,8 @@ SIGNATURES = {
     "nest_datastore_reserve": (ctypes.c_int, [_P, _I32, _I32, _I32]),
     "nest_datastore_use_cta_pairs": (ctypes.c_int, [_P, _I32]),
     "nest_selftest_bounded_wait": (ctypes.c_int, [_P, ctypes.POINTER(_I64), _P]),
+    "nest_plan_offline": (ctypes.c_int, [_I64, _I32, _I32, _I32, _I32, _I32, _I32, _I64, _I32,
+                                         _P]),
     "nest_knn_search": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_static": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P]),
     "nest_knn_search_masked": (ctypes.c_int, [_P, _P, _I32, _I32, _P, _P, _P, _P, _P]),
@@ -56,6 +58,15 @@ SIGNATURES = {
 }
 
 _lib = None
+
+
+class Plan(ctypes.Structure):
+    """nest_plan_t (include/nest.h)."""
+    _fields_ = [("path", ctypes.c_int32), ("queries_per_group", ctypes.c_int32),
+                ("groups", ctypes.c_int32), ("parts", ctypes.c_int32),
+                ("stages", ctypes.c_int32), ("single_pass", ctypes.c_int32),
+                ("sample_stride", ctypes.c_int64), ("list_capacity", ctypes.c_int64),
+                ("scratch_bytes", ctypes.c_int64)]
 
 
 class NestError(RuntimeError):
@@ -81,6 +92,25 @@ def load_library(path: str | None = None):
     if path is None:
         _lib = lib
     return lib
+
+
+def plan_offline(N: int, d: int, dtype: str, B: int, r: int, ragged: bool = False,
+                 num_sms: int = 152, smem_per_block: int = 232448,
+                 cta_pairs: bool = False) -> dict:
+    """The plan a search of this shape would run (nest_plan_offline): host
+    only, no GPU.  The defaults are a GB300's 152 SMs and 227 KiB of opt-in
+    shared memory per block.  ``dtype`` is "f32" or "bf16"."""
+    lib = load_library()
+    p = Plan()
+    code = BF16 if dtype == "bf16" else F32 if dtype == "f32" else -1
+    if code < 0:
+        raise ValueError("dtype must be 'f32' or 'bf16'")
+    _check(lib.nest_plan_offline(int(N), int(d), code, int(B), int(r), int(bool(ragged)),
+                                 int(num_sms), int(smem_per_block), int(bool(cta_pairs)),
+                                 ctypes.byref(p)), "nest_plan_offline")
+    out = {name: getattr(p, name) for name, _ in Plan._fields_}
+    out["kernel"] = Datastore.SEARCH_PATHS[p.path]
+    return out
 
 
 def _check(code: int, where: str) -> None:

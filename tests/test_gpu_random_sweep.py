@@ -256,16 +256,26 @@ def _run_case(nest, c):
 
 
 def test_sweep_reaches_every_search_path(nest):
-    """The drawn shapes run every distance-scan kernel the library has."""
+    """The drawn shapes run every distance-scan kernel the library has, and a
+    handle on this device picks the kernel nest_plan_offline predicts from
+    the device's SM count and shared memory per block."""
     seen = set()
+    props = torch.cuda.get_device_properties(0)
+    smem = getattr(props, "shared_memory_per_block_optin", None)
     V = torch.zeros(64, dtype=torch.int32, device="cuda")
     for c in CASES + EDGE_CASES:
         K = torch.zeros(64, c["d"], dtype=synth.torch_dtype(c["dtype"]), device="cuda")
         ds = nest.Datastore(K, V, 10)
         if _pairs(c):
             ds.use_cta_pairs(True)
-        seen.add(ds.search_path(c["B"], c["r"], ragged=c["ragged"]))
+        path = ds.search_path(c["B"], c["r"], ragged=c["ragged"])
+        seen.add(path)
         ds.close()
+        if smem:
+            plan = nest.plan_offline(64, c["d"], c["dtype"], c["B"], c["r"], ragged=c["ragged"],
+                                     num_sms=props.multi_processor_count, smem_per_block=smem,
+                                     cta_pairs=_pairs(c))
+            assert plan["kernel"] == path, (c, plan)
     assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
                     "tc_wide_pair_kernel", "scan_topr_kernel"}, seen
 

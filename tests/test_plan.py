@@ -1,0 +1,133 @@
+"""The search planner on a machine without a GPU (nest_plan_offline).
+
+nest_plan_offline runs the planning code of nest_knn_search for a given
+datastore shape and device (SM count, shared memory per block), so the host
+logic that picks the kernel, splits the work and sizes the scratch is
+checked here without a GPU:
+  * the benchmarked workloads get the plans their descriptions state (one
+    wave of CTAs on 152 SMs, the 65,536-key threshold sample, the static
+    array's 8 MiB budget for the decode search);
+  * every shape of the GPU sweeps satisfies the planner's invariants (all
+    queries covered, lists with room for a tile of appends, samples of at
+    least 65,536 keys, scratch for every list);
+  * arguments are checked as nest_datastore_create / nest_knn_search check
+    them.
+"""
+import os
+import sys
+
+import pytest
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+SMS, SMEM = 152, 232448  # a GB300: 152 SMs, 227 KiB opt-in shared memory per block
+
+
+@pytest.fixture(scope="module")
+def nest():
+    from paper_2405_19325_gb300 import build as nest_build
+    nest_build.build()
+    import paper_2405_19325_gb300 as pkg
+    pkg.load_library()
+    return pkg
+
+
+def test_decode_plan(nest):
+    """B=4, 1M bf16 keys of 4096, r=1024: the narrow tensor-core scan, one
+    group of 4 queries over 152 key ranges (one CTA per SM), scratch within
+    the allocation-free entry point's 2^20 words."""
+    p = nest.plan_offline(1 << 20, 4096, "bf16", 4, 1024, num_sms=SMS, smem_per_block=SMEM)
+    assert p["kernel"] == "tc_scan_kernel"
+    assert (p["queries_per_group"], p["groups"], p["parts"]) == (4, 1, SMS)
+    assert p["list_capacity"] >= 1024 + 128
+    assert p["scratch_bytes"] <= (1 << 20) * 8
+
+
+def test_large_batch_plan(nest):
+    """B=512, 4M keys, r=256: two groups of 256 queries, every key range once
+    per group in one wave (2 x 76 CTAs), thresholds from every 64th key
+    (65,536 = max(65,536, 256 r) sampled keys)."""
+    p = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM)
+    assert p["kernel"] == "tc_wide2_kernel"
+    assert (p["queries_per_group"], p["groups"], p["parts"]) == (256, 2, SMS // 2)
+    assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // 65536
+    assert p["list_capacity"] >= 8 * ((1 << 22) * 256 // 65536)  # 8x the expected survivors
+    q = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
+                          cta_pairs=True)
+    assert q["kernel"] == "tc_wide_pair_kernel"
+    assert (q["groups"], q["parts"]) == (2, SMS // 4)  # 2 groups x 38 pairs = 152 SMs
+
+
+def test_ragged_and_fp32_plans(nest):
+    p = nest.plan_offline(32 * 10240, 4096, "bf16", 32, 64, ragged=True, num_sms=SMS,
+                          smem_per_block=SMEM)
+    assert p["kernel"] == "tc_scan_kernel"
+    assert (p["queries_per_group"], p["groups"]) == (1, 32)  # one query per CTA, own segment
+    p = nest.plan_offline(4096, 64, "f32", 8, 16, num_sms=SMS, smem_per_block=SMEM)
+    assert p["kernel"] == "scan_topr_kernel"
+
+
+def test_large_batch_single_pass_when_the_sample_is_every_key(nest):
+    p = nest.plan_offline(60000, 256, "bf16", 300, 64, num_sms=SMS, smem_per_block=SMEM)
+    assert p["single_pass"] == 1 and p["sample_stride"] == 1
+    assert p["list_capacity"] == 60000  # every key's word at its row position
+
+
+def _sweep_shapes():
+    import test_gpu_random_sweep as sweep
+    return sweep.CASES + sweep.EDGE_CASES, sweep._pairs
+
+
+def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
+    cases, pairs_of = _sweep_shapes()
+    seen = set()
+    for c in cases:
+        N, d, B, r = c["N"], c["d"], c["B"], c["r"]
+        p = nest.plan_offline(N, d, c["dtype"], B, r, ragged=c["ragged"], num_sms=SMS,
+                              smem_per_block=SMEM, cta_pairs=pairs_of(c))
+        seen.add(p["kernel"])
+        tag = f"{c}: {p}"
+        qpg, groups = p["queries_per_group"], p["groups"]
+        # the smallest ring each kernel is planned with
+        assert p["parts"] >= 1 and p["stages"] >= {0: 2, 1: 4, 2: 3, 3: 3, 4: 4}[p["path"]], tag
+        assert (c["dtype"] == "f32") == (p["path"] == 0), tag
+        if c["ragged"]:
+            assert qpg == 1 and groups == B, tag
+        else:
+            assert groups * qpg >= B > (groups - 1) * qpg, tag
+        if p["path"] <= 1:
+            # room for a list of r plus the appends of at least one block of keys
+            assert p["list_capacity"] > r, tag
+            assert p["scratch_bytes"] >= groups * p["parts"] * qpg * r * 8, tag
+        else:
+            assert not c["ragged"] and c["dtype"] == "bf16", tag
+            assert (p["path"] == 4) == (pairs_of(c) and qpg == 256), tag
+            if p["single_pass"]:
+                assert p["sample_stride"] == 1 and p["list_capacity"] == N, tag
+            else:
+                k = 256 if qpg == 256 else 64
+                target = max(65536, k * r)
+                assert p["sample_stride"] == N // target >= 2, tag
+                assert N // p["sample_stride"] >= target, tag
+                assert p["list_capacity"] >= min(N, 8 * r), tag
+            assert p["scratch_bytes"] >= B * p["list_capacity"] * 8, tag
+    assert seen >= {"scan_topr_kernel", "tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
+                    "tc_wide_pair_kernel"}, seen
+
+
+def test_plan_argument_checks(nest):
+    from paper_2405_19325_gb300 import NestError
+    bad = [
+        (dict(N=0, d=64, dtype="f32", B=1, r=1), 1),
+        (dict(N=10, d=3, dtype="f32", B=1, r=1), 3),        # 12-byte rows
+        (dict(N=10, d=8200, dtype="bf16", B=1, r=1), 9),    # row above NEST_MAX_ROW_BYTES
+        (dict(N=10, d=64, dtype="f32", B=0, r=1), 1),
+        (dict(N=10, d=64, dtype="f32", B=65536, r=1), 1),
+        (dict(N=10, d=64, dtype="f32", B=1, r=4097), 1),
+    ]
+    for kw, code in bad:
+        with pytest.raises(NestError) as e:
+            nest.plan_offline(**kw, num_sms=SMS, smem_per_block=SMEM)
+        assert e.value.code == code, kw
+    with pytest.raises(ValueError):
+        nest.plan_offline(10, 64, "f16", 1, 1)
