@@ -458,6 +458,19 @@ def test_wide_batch_massive_exact_ties(nest, pairs):
                   pairs=pairs)
 
 
+@pytest.mark.parametrize("N,d,B,r", [
+    (200000, 128, 2048, 64),   # 8 query groups over 19 key ranges, two passes
+    (70017, 64, 4000, 33),     # 16 groups (the last one partial), one pass
+])
+def test_many_query_groups(nest, N, d, B, r):
+    """Batches far above 256 queries: many groups of 256 stream each key
+    range (adjacent CTAs share its tiles in L2), and every group's lists,
+    counters and thresholds stay separate.  Rows sampled across all groups."""
+    K, V, q, p_lm = _random_case(N, d, B, 600, "bf16", seed=B + r, centres=40)
+    rows = sorted(set(list(range(0, B, B // 12)) + [255, 256, B - 1]))
+    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, 600, "bf16", check_rows=rows)
+
+
 def test_large_batch_shape_sampled_rows(nest):
     """Large-batch shape: bf16 d=4096, B=512, r=256, clustered keys (N reduced
     to 524,288); the oracle checks 12 query rows spread over the batch."""
