@@ -1,6 +1,7 @@
 // api.cu -- the C ABI of include/nest.h: argument validation, the datastore
 // handle, scratch memory, and the choice and launch of the kernels.
 #include <algorithm>
+#include <cstdint>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -211,11 +212,15 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             sp->off_i_s = sp->off_s_s + ((size_t)B * r + 1) / 2;
             sp->off_cand_m = sp->off_i_s + (size_t)B * r;
             sp->wide_words = sp->single_pass ? sp->off_s_s : sp->off_cand_m + (size_t)B * sp->cap_m;
-            sp->wide = true;
-            sp->cand_words = sp->wide_words;
-            sp->level_words = 0;
-            sp->cnt_words = 0;
-            sp->total_words = sp->wide_words;
+            // list positions and counters are 32-bit in the kernels: lists
+            // that could pass 2^31 words stay on the narrow scan
+            if (sp->cap_s < INT32_MAX && (sp->single_pass || sp->cap_m < INT32_MAX)) {
+                sp->wide = true;
+                sp->cand_words = sp->wide_words;
+                sp->level_words = 0;
+                sp->cnt_words = 0;
+                sp->total_words = sp->wide_words;
+            }
         }
     }
     return NEST_OK;

@@ -131,3 +131,16 @@ def test_plan_argument_checks(nest):
         assert e.value.code == code, kw
     with pytest.raises(ValueError):
         nest.plan_offline(10, 64, "f16", 1, 1)
+
+
+def test_largest_tensor_core_datastore_keeps_32_bit_lists(nest):
+    """At the largest bf16 datastore the tensor-core paths take (0x7FFFFF00
+    keys), every list the large-batch kernels index with 32-bit positions
+    stays below 2^31 words: samples hold at least 64 r keys, so a query's
+    survivors are at most about N / 8 plus the reservation blocks."""
+    N = 0x7FFFFF00
+    for B, r in [(17, 1), (64, 1024), (512, 4096)]:
+        p = nest.plan_offline(N, 8, "bf16", B, r, num_sms=SMS, smem_per_block=SMEM)
+        assert p["path"] in (2, 3), p
+        assert p["list_capacity"] < 2 ** 31, p
+        assert p["list_capacity"] <= N // 8 + p["parts"] * 8 * 1024, p
