@@ -3,7 +3,8 @@
 // query row.
 //
 // Grid (slices, B).  Every CTA of a row reads the row's r neighbours,
-// gathers their token ids V[idx], and forms the softmax weights
+// gathers their token ids V[idx] once into shared memory, and forms the
+// softmax weights
 // w_i = exp(mu (s_i - s_max)) / Z.  Weights of tokens inside the CTA's
 // vocabulary slice are summed per token in shared memory as 48-bit fixed
 // point: integer addition is associative, so the sums do not depend on the
@@ -51,7 +52,12 @@ __device__ __forceinline__ float warp_min(float x)
 
 __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
 {
-    extern __shared__ __align__(16) unsigned long long acc[];  // slice tokens, fixed point
+    // The row's neighbours, gathered once (token id, -1 for no weight; s),
+    // then the slice's fixed-point sums.
+    extern __shared__ __align__(16) unsigned long long smem_mix[];
+    int32_t* tok = reinterpret_cast<int32_t*>(smem_mix);
+    float* sim = reinterpret_cast<float*>(tok + a.r);
+    unsigned long long* acc = smem_mix + a.r;
     __shared__ Red red;
     __shared__ float bc[4];
     __shared__ int bci;
@@ -74,16 +80,19 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
     for (int i = tid; i < a.r; i += kMixThreads) {
         const int64_t k = id[i];
         const float si = s[i];
-        if (k < 0 || !(si > -INFINITY)) continue;
-        if (k >= a.N) {
-            record_status(a.status, NEST_ERR_VALUE_RANGE);
-            continue;
+        int32_t v = -1;
+        if (k >= 0 && si > -INFINITY) {
+            if (k >= a.N) {
+                record_status(a.status, NEST_ERR_VALUE_RANGE);
+            } else {
+                const int32_t t = a.V[k];
+                if (t < 0 || t >= a.vocab) record_status(a.status, NEST_ERR_VALUE_RANGE);
+                else v = t;
+            }
         }
-        const int32_t v = a.V[k];
-        if (v < 0 || v >= a.vocab) {
-            record_status(a.status, NEST_ERR_VALUE_RANGE);
-            continue;
-        }
+        tok[i] = v;  // each thread reads back only the entries it wrote
+        sim[i] = si;
+        if (v < 0) continue;
         smax = fmaxf(smax, si);
         amin = fminf(amin, fabsf(si));
         amax = fmaxf(amax, fabsf(si));
@@ -122,12 +131,8 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
     // Z = sum of exp(mu (s_i - s_max)) over real neighbours (fixed-order tree).
     float zpart = 0.f;
     for (int i = tid; i < a.r; i += kMixThreads) {
-        const int64_t k = id[i];
-        const float si = s[i];
-        if (k < 0 || k >= a.N || !(si > -INFINITY)) continue;
-        const int32_t v = a.V[k];
-        if (v < 0 || v >= a.vocab) continue;
-        zpart += expf(a.mu * (si - smax));
+        if (tok[i] < 0) continue;
+        zpart += expf(a.mu * (sim[i] - smax));
     }
     zpart = warp_sum(zpart);
     if (lane == 0) red.v[warp] = zpart;
@@ -151,12 +156,9 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
 
     // p_kNN of the slice's tokens: w_i / Z summed per token in fixed point.
     for (int i = tid; i < a.r; i += kMixThreads) {
-        const int64_t k = id[i];
-        const float si = s[i];
-        if (k < 0 || k >= a.N || !(si > -INFINITY)) continue;
-        const int32_t v = a.V[k];
-        if (v < w0 || v >= w1) continue;
-        const float p = expf(a.mu * (si - smax)) / z;
+        const int32_t v = tok[i];
+        if (v < w0 || v >= w1) continue;  // also skips v = -1 (w0 >= 0)
+        const float p = expf(a.mu * (sim[i] - smax)) / z;
         atomicAdd(&acc[v - w0], (unsigned long long)__float2ull_rn(p * kFixScale));
     }
     __syncthreads();
@@ -202,7 +204,8 @@ cudaError_t launch_mix(const MixArgs& a, cudaStream_t stream)
     const int unit = (a.vocab & 3) == 0 ? 4 : 1;
     const int64_t units = a.vocab / unit;
     const int widest = unit * (int)((units + a.slices - 1) / a.slices) + unit;
-    const size_t smem = (size_t)widest * sizeof(unsigned long long);
+    // r gathered neighbours (token id and s, 8 bytes) + the slice's sums
+    const size_t smem = ((size_t)a.r + widest) * sizeof(unsigned long long);
     cudaError_t e =
         raise_smem_limit(reinterpret_cast<const void*>(mix_kernel), (int)smem);
     if (e != cudaSuccess) return e;
