@@ -44,3 +44,22 @@ def test_cuda_arm_refuses_to_run_without_a_gpu():
     assert res.returncode != 0
     assert not [l for l in res.stdout.splitlines() if l.startswith("{")]
     assert "CUDA" in (res.stdout + res.stderr)
+
+
+def test_reference_arm_under_torchrun_prints_once():
+    """Launched as the driver launches N ranks: rank 0 alone runs the oracle
+    and prints the line; the other rank exits 0 without work."""
+    import socket
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    res = subprocess.run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+                          "--nproc-per-node", "2", "--master-addr", "127.0.0.1",
+                          "--master-port", str(port), os.path.join(ROOT, "bench.py"),
+                          "--impl", "reference", "--workload", "tiny", "--steps", "1",
+                          "--warmup", "1"], cwd=ROOT, capture_output=True, text=True,
+                         timeout=300)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    assert json.loads(lines[0])["impl"] == "reference"
