@@ -110,6 +110,25 @@ def test_topr_brute_force_with_ties(r):
         assert np.all(idx[b, n:] == -1) and np.all(np.isneginf(s[b, n:]))
 
 
+def test_chunked_search_matches_brute_force_in_any_chunk_order():
+    """knn_search_chunked (keys delivered in pieces, as the full-size d=8192
+    parity test streams them back from the device) against a brute-force
+    sort: uneven chunks in shuffled order, integer keys with many ties."""
+    rng = np.random.default_rng(21)
+    K = rng.integers(-2, 3, size=(257, 5)).astype(np.float32)
+    q = rng.integers(-2, 3, size=(3, 5)).astype(np.float32)
+    cuts = [0, 1, 64, 65, 200, 257]
+    chunks = [(cuts[i], K[cuts[i]:cuts[i + 1]]) for i in range(len(cuts) - 1)]
+    order = rng.permutation(len(chunks))
+    r = 40
+    s, idx = oracle.knn_search_chunked([chunks[i] for i in order], q, r)
+    D = cdist(q.astype(np.float64), K.astype(np.float64), "sqeuclidean")
+    for b in range(3):
+        want = _brute_topr(D[b], r)
+        assert idx[b].tolist() == [i for _, i in want]
+        assert (-s[b]).tolist() == [dd for dd, _ in want]
+
+
 def test_topr_r_equals_n_returns_every_key_sorted():
     rng = np.random.default_rng(6)
     K = rng.standard_normal((40, 8)).astype(np.float32)
