@@ -32,6 +32,15 @@ MUTANTS = {
     "verify_without_gamma": ("ratio[b] = mx > 0.0 ? p / (gamma * mx) : 0.0;",
                              "ratio[b] = mx > 0.0 ? p / mx : 0.0;"),
     "verify_accepts_half": ("accept[b] = a > 0.5 ? 1 : 0;", "accept[b] = a >= 0.5 ? 1 : 0;"),
+    "rrc_sigmoid_sign": ("return 1.0 / (1.0 + exp(-(ratio - alpha) / tau));",
+                         "return 1.0 / (1.0 + exp((ratio - alpha) / tau));"),
+    "rrc_ratio_inverted": ("double ratio = (hi == 0.0) ? 1.0 : lo / hi;",
+                           "double ratio = (lo == 0.0) ? 1.0 : hi / lo;"),
+    "rrc_counts_padding": ("        if (idx[i] < 0) continue;\n        double a = fabs(s[i]);",
+                           "        double a = fabs(s[i]);"),
+    "verify_counts_past_a_rejection": (
+        "while (span_off[j] + n < span_off[j + 1] && accept[span_off[j] + n]) ++n;",
+        "for (int32_t t = span_off[j]; t < span_off[j + 1]; ++t) n += accept[t];"),
 }
 
 
