@@ -97,6 +97,42 @@ def test_search_and_mix_validation(lib):
     assert lib.nest_knn_step(ds, q, 1, 1, None, p, 1.0, 0.5, None, i, None, p, None) == 1
 
 
+def test_nest_step_calls_validation(lib):
+    """The decision, verification, masking and diagnostic calls refuse bad
+    arguments on the host, before they touch the handle or the device."""
+    P = ctypes.c_void_p
+    ds, a = P(FAKE), P(FAKE)
+    # masked search: the mask is required and 4-byte aligned
+    assert lib.nest_knn_search_masked(None, a, 1, 1, None, None, a, a, None) == 1
+    assert lib.nest_knn_search_masked(ds, a, 1, 1, None, None, a, a, None) == 1
+    assert lib.nest_knn_search_masked(ds, a, 1, 1, None, P(FAKE + 2), a, a, None) == 3
+    # masking: a negative start or count
+    assert lib.nest_mask_keys(None, a, 0, 1, None) == 1
+    assert lib.nest_mask_keys(ds, a, -1, 1, None) == 1
+    assert lib.nest_mask_keys(ds, a, 0, -1, None) == 1
+    # Eq. 5 / Eq. 6
+    args = [a] * 4
+    assert lib.nest_knn_decide(None, a, a, a, a, 1, 1, 0.5, *args, None) == 1
+    assert lib.nest_knn_decide(ds, a, a, a, a, 0, 1, 0.5, *args, None) == 1
+    assert lib.nest_knn_decide(ds, a, a, a, a, 1, 4097, 0.5, *args, None) == 1
+    assert lib.nest_knn_decide(ds, a, a, a, a, 1, 1, float("nan"), *args, None) == 1
+    assert lib.nest_knn_decide(ds, a, a, P(FAKE + 4), a, 1, 1, 0.5, *args, None) == 3
+    # Eq. 7: rows, spans and gamma
+    assert lib.nest_verify_spans(None, a, a, 1, a, 1, 0.5, a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, a, a, 0, a, 1, 0.5, a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, a, a, 1, a, 0, 0.5, a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, a, a, 70000, a, 1, 0.5, a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, a, a, 1, a, 1, 0.0, a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, a, a, 1, a, 1, float("nan"), a, a, a, None) == 1
+    assert lib.nest_verify_spans(ds, P(FAKE + 2), a, 1, a, 1, 0.5, a, a, a, None) == 3
+    # handle-level calls
+    assert lib.nest_datastore_use_cta_pairs(None, 1) == 1
+    assert lib.nest_selftest_bounded_wait(None, None, None) == 1
+    assert lib.nest_datastore_reserve(None, 1, 1, 0) == 1
+    assert lib.nest_search_path(None, 1, 1, 0) == -1
+    assert lib.nest_datastore_destroy(None) == 0
+
+
 def test_no_cpu_fallback_when_library_missing():
     from paper_2405_19325_gb300 import nest
     with pytest.raises(RuntimeError):
