@@ -59,7 +59,8 @@ typedef enum nest_status {
     NEST_ERR_VALUE_RANGE = 6,  /* token id outside [0, vocab) or key index outside [0, N) */
     NEST_ERR_OVERFLOW = 7,     /* a search needs more than a fixed-size scratch buffer holds */
     NEST_ERR_TIMEOUT = 8,      /* a device-side wait gave up */
-    NEST_ERR_UNSUPPORTED = 9   /* shape outside what the kernels handle */
+    NEST_ERR_UNSUPPORTED = 9,  /* shape outside what the kernels handle */
+    NEST_ERR_MARGIN = 10       /* exact re-ranking could not confirm a query's r-th neighbour */
 } nest_status_t;
 
 typedef enum nest_dtype { NEST_F32 = 0, NEST_BF16 = 1 } nest_dtype_t;
@@ -139,8 +140,20 @@ NEST_API nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_
  *   idx_out  B x r int64 global key indices of the neighbours.
  *
  * When a query has fewer than r candidate keys the tail of its row is
- * padded with s = -inf and idx = -1.  Distances are evaluated as
- * ||q||^2 + ||k||^2 - 2 q.k in fp32 and clamped at 0.
+ * padded with s = -inf and idx = -1.
+ *
+ * Distances: every key is screened by ||q||^2 + ||k||^2 - 2 q.k evaluated in
+ * fp32 (tensor cores for bf16 keys), whose rounding error is absolute in the
+ * norms.  Each query keeps its r' = r + m nearest screened keys
+ * (m = r / 16, at least 16 and at most 128), their distances are recomputed
+ * as sums of squared differences of the stored elements in fp32 (error a
+ * few units in the last place of the distance itself; exactly 0 for a key
+ * equal to the query), and the r nearest by those are returned.  If more
+ * than m keys lie within the screening error of the r-th distance, a key
+ * outside the r' might belong to the r nearest: this is detected from the
+ * screening errors seen among the r' (see refine.cu) and recorded as
+ * NEST_ERR_MARGIN in the device status; the row then holds the r nearest of
+ * the r' candidates.
  */
 NEST_API nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
                               const int64_t* seg_off, float* s_out, int64_t* idx_out,
@@ -241,9 +254,10 @@ NEST_API nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_
  * (ordered with `stream` by events), so those copies overlap the search and
  * the mix.  The device buffers grow on demand with cudaMalloc, the side
  * stream is created on the first call, and nest_datastore_destroy frees
- * both; calls on one handle must not overlap.  Device-side
- * errors of the kernels are reported by nest_device_status, as for
- * nest_knn_step.  The paper's method is the same as nest_knn_step (Eq. 1-3);
+ * both; calls on one handle must not overlap.  The call also reads the
+ * device status word once the step is done and returns the first condition
+ * the kernels recorded (clearing it, as nest_device_status does), so an
+ * overflow or a failed margin check is never returned as NEST_OK.  The paper's method is the same as nest_knn_step (Eq. 1-3);
  * only the data movement differs.
  */
 NEST_API nest_status_t nest_knn_step_host(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,

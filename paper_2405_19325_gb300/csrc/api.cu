@@ -38,6 +38,7 @@ struct nest_datastore {
     size_t host_stage_bytes = 0;
     cudaStream_t aux = nullptr;           // owned: side stream of nest_knn_step_host
     cudaEvent_t aux_ev[3] = {nullptr, nullptr, nullptr};
+    int* host_status = nullptr;           // owned, page-locked: status copy of nest_knn_step_host
     bool timing = false;
     std::vector<cudaEvent_t> events;  // pairs (start, end)
     size_t events_used = 0;
@@ -47,6 +48,9 @@ struct nest_datastore {
 namespace {
 
 constexpr int64_t kMaxKeys = 4294967294LL;  // key indices travel as 32 bits
+// Recovery passes after an overflowed large-batch list (each at most one
+// more scan of the keys, only for the query groups concerned).
+constexpr int kRecoverRounds = 2;
 constexpr int32_t kMaxB = 65535;
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -65,23 +69,28 @@ int element_size(int dtype) { return dtype == NEST_BF16 ? 2 : 4; }
 // Search layout chosen for a call: which scan kernel, its plan, and the
 // candidate words of the scan output and of the merge levels.
 struct SearchPlan {
+    int r;         // neighbours returned
+    int rp;        // screened candidates kept per query for the exact re-ranking
     bool tc;       // tensor-core scan (bf16) or CUDA-core scan
     ScanPlan scan;
     TcPlan tcp;
     int nq, groups, parts;
-    size_t cand_words;   // scan output: groups * parts * nq * r
+    size_t cand_words;   // scan output: groups * parts * nq * rp
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
     size_t cnt_words;    // list lengths of the scan output and of the merge levels
+    size_t off_fin;      // each query's rp candidates for the re-ranking: B * rp words,
+                         // B int32 lengths and 3 * B uint32 of re-ranking state (rounded
+                         // up to whole words), then B 64-bit words of state
     size_t total_words;  // all scratch of the search
     // Large query batches (tc_wide.cu): sample pass + thresholded pass.
     bool wide;
-    WidePlan wps, wpm;        // sample pass, main pass
+    WidePlan wps, wpm, wpr;   // sample pass, main pass, recovery pass
     int64_t stride;           // sample = every stride-th key
     int64_t sample_rows;
     bool single_pass;         // the sample is the whole datastore
     int64_t cap_s, cap_m;     // list capacities per query
     int32_t resv;             // main pass: list slots an epilogue warp reserves at a time
-    size_t off_cnt, off_qn, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
+    size_t off_cnt, off_qn, off_lim, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
 };
 
 // Parts per query group.  Time ~ waves * (work per part + fixed cost per part),
@@ -113,8 +122,15 @@ int ceil_pow2(int x)
     return p;
 }
 
-nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, SearchPlan* sp)
+nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragged,
+                          SearchPlan* sp)
 {
+    // Every step below keeps r = r_out + margin screened candidates; the
+    // exact re-ranking (refine.cu) returns r_out of them.
+    const int r = r_out + refine_margin(r_out);
+    sp->r = r_out;
+    sp->rp = r;
+    const size_t fin_words = (size_t)B * r + ((size_t)4 * B + 1) / 2 + (size_t)B;
     sp->tc = false;
     const int64_t keys_per_group_full = ds->N;
     if (ds->tc) {
@@ -163,7 +179,8 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
     // int32 counts: [groups * parts * nq] then [B * lvl1], as 64-bit words
     sp->cnt_words = ((size_t)sp->groups * sp->parts * sp->nq + 1) / 2 + ((size_t)B * lvl1 + 1) / 2;
-    sp->total_words = sp->cand_words + sp->level_words + sp->cnt_words;
+    sp->off_fin = sp->cand_words + sp->level_words + sp->cnt_words;
+    sp->total_words = sp->off_fin + fin_words;
     sp->wide = false;
     // More queries than one CTA can keep lists for: stream the keys once per
     // group of up to 256 queries against sampled admission thresholds.
@@ -205,9 +222,16 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
             sp->resv = (int32_t)std::min<int64_t>(2 * per_warp + 16, 1024);
             const int64_t unwritten = (int64_t)sp->wpm.parts * epi_warps * sp->resv;
             sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect)) + unwritten;
-            sp->off_cnt = 0;  // 2 * B int32 counters
-            sp->off_qn = (size_t)B;  // B floats: ||q||^2
-            sp->off_cand_s = sp->off_qn + ((size_t)B + 1) / 2;
+            // recovery of overflowed main-pass lists: the same groups, one
+            // 128-key tile per stage
+            if (!wide_recover_plan(nm, ds->smem_optin, &sp->wpr)) return NEST_ERR_UNSUPPORTED;
+            sp->wpr.groups = wp.groups;
+            sp->wpr.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
+            // 2 * B int32 counters, then kRecoverRounds * groups int32 flags
+            sp->off_cnt = 0;
+            sp->off_qn = (2 * (size_t)B + (size_t)kRecoverRounds * wp.groups + 1) / 2;
+            sp->off_lim = sp->off_qn + ((size_t)B + 1) / 2;  // after B floats ||q||^2
+            sp->off_cand_s = sp->off_lim + (size_t)B;       // after B word limits
             sp->off_s_s = sp->off_cand_s + (size_t)B * sp->cap_s;
             sp->off_i_s = sp->off_s_s + ((size_t)B * r + 1) / 2;
             sp->off_cand_m = sp->off_i_s + (size_t)B * r;
@@ -219,7 +243,8 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r, bool ragged, S
                 sp->cand_words = sp->wide_words;
                 sp->level_words = 0;
                 sp->cnt_words = 0;
-                sp->total_words = sp->wide_words;
+                sp->off_fin = sp->wide_words;
+                sp->total_words = sp->wide_words + fin_words;
             }
         }
     }
@@ -342,13 +367,17 @@ nest_status_t ensure_host_stage(nest_datastore* ds, size_t bytes)
 
 size_t round256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-// The side stream and events of nest_knn_step_host, created on first use.
+// The side stream, events and page-locked status word of
+// nest_knn_step_host, created on first use.
 nest_status_t ensure_aux(nest_datastore* ds)
 {
     if (ds->aux) return NEST_OK;
     cudaError_t e = cudaStreamCreateWithFlags(&ds->aux, cudaStreamNonBlocking);
     for (int i = 0; i < 3 && e == cudaSuccess; ++i)
         e = cudaEventCreateWithFlags(&ds->aux_ev[i], cudaEventDisableTiming);
+    if (e == cudaSuccess && !ds->host_status)
+        e = cudaHostAlloc(reinterpret_cast<void**>(&ds->host_status), sizeof(int),
+                          cudaHostAllocDefault);
     if (e != cudaSuccess) {
         for (cudaEvent_t& ev : ds->aux_ev) {
             if (ev) (void)cudaEventDestroy(ev);
@@ -383,6 +412,18 @@ nest_status_t check_search_args(const nest_datastore* ds, const void* q, int32_t
     return NEST_OK;
 }
 
+// Kernels run on the current device and read the datastore's memory: a call
+// made with another device current is refused before anything is launched.
+nest_status_t check_device(const nest_datastore* ds)
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return NEST_ERR_CUDA;
+    }
+    return dev == ds->device ? NEST_OK : NEST_ERR_INVALID_ARG;
+}
+
 nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const int64_t* idx_in,
                              const float* p_lm, int32_t B, int32_t r, const float* p_knn_out,
                              const float* p_m_out)
@@ -396,14 +437,19 @@ nest_status_t check_mix_args(const nest_datastore* ds, const float* s_in, const 
 }
 
 // Large query batches: [sample pass, selection of the sample,] thresholded
-// pass over all keys, exact selection of the survivors.
+// pass over all keys, selection of each query's rp candidates into the
+// re-ranking region (fin, fin_cnt, state).
 nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* q, int32_t B,
-                          int32_t r, const uint32_t* key_mask, float* s_out, int64_t* idx_out,
-                          uint64_t* scratch, bool timed, cudaStream_t stream)
+                          const uint32_t* key_mask, uint64_t* scratch, uint64_t* fin,
+                          int32_t* fin_cnt, uint32_t* state, unsigned long long* apair,
+                          bool timed, cudaStream_t stream)
 {
+    const int32_t r = sp.rp;
     nest_status_t st;
     int32_t* cnt = reinterpret_cast<int32_t*>(scratch + sp.off_cnt);
-    cudaError_t e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * 2 * (size_t)B, stream);
+    int32_t* flags = cnt + 2 * (size_t)B;  // kRecoverRounds rows of groups
+    cudaError_t e = cudaMemsetAsync(
+        cnt, 0, sizeof(int32_t) * (2 * (size_t)B + (size_t)kRecoverRounds * sp.wpm.groups), stream);
     if (e != cudaSuccess) return from_cuda(e);
     CUtensorMap qmap;
     // a CTA of a pair stages half of the group's queries
@@ -432,7 +478,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     ga.B = B;
 
     if (sp.single_pass) {
-        // the "sample" is every key: its exact r nearest are the answer
+        // the "sample" is every key: its r nearest screened are the candidates
         wa.s_sample = nullptr;
         wa.cand = scratch + sp.off_cand_s;
         wa.cnt = cnt;
@@ -447,8 +493,10 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
         ga.cand = wa.cand;
         ga.cnt = cnt;
         ga.cap = sp.cap_s;
-        ga.s_out = s_out;
-        ga.idx_out = idx_out;
+        ga.words_out = fin;
+        ga.words_cnt = fin_cnt;
+        ga.refine_state = state;
+        ga.refine_apair = apair;
         e = launch_gselect(ga, stream);
         if (e != cudaSuccess) return from_cuda(e);
         ds->launches += 2;
@@ -477,7 +525,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     ga.idx_out = i_s;
     e = launch_gselect(ga, stream);
     if (e != cudaSuccess) return from_cuda(e);
-    // 2. every key, admitted at or below the sample's r-th distance
+    // 2. every key, admitted at or below the sample's r-th screened distance
     wa.s_sample = s_s;
     wa.cand = scratch + sp.off_cand_m;
     wa.cnt = cnt + B;
@@ -490,113 +538,175 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
     if (e != cudaSuccess) return from_cuda(e);
     if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+    // 3. lists that overflowed (more survivors than their capacity: many
+    // keys tied at the sample's threshold, say) are scanned again with a
+    // tighter limit: the r-th smallest word each holds.  Both kernels of a
+    // round return at once when no list needs it.
+    uint64_t* lim = scratch + sp.off_lim;
+    CUtensorMap rmap;
+    if (!encode_bf16_rows(&rmap, q, B, ds->d, sp.wpr.nm, false)) return NEST_ERR_CUDA;
+    for (int round = 0; round < kRecoverRounds; ++round) {
+        GselectArgs gp{};
+        gp.cand = wa.cand;
+        gp.cnt = cnt + B;
+        gp.cap = sp.cap_m;
+        gp.r = r;
+        gp.B = B;
+        gp.lim_out = lim;
+        gp.group_flag = flags + (size_t)round * sp.wpm.groups;
+        gp.group_size = sp.wpm.nm;
+        e = launch_gselect(gp, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        WideArgs wr = wa;
+        wr.resv = 0;
+        wr.parts = sp.wpr.parts;
+        wr.stages = sp.wpr.stages;
+        wr.word_lim = lim;
+        wr.group_flag = gp.group_flag;
+        e = launch_tc_wide_recover(sp.wpr, ds->keys_map, rmap, wr, stream);
+        if (e != cudaSuccess) return from_cuda(e);
+        ds->launches += 2;
+    }
     ga.cand = wa.cand;
     ga.cnt = cnt + B;
     ga.cap = sp.cap_m;
-    ga.s_out = s_out;
-    ga.idx_out = idx_out;
+    ga.s_out = nullptr;
+    ga.idx_out = nullptr;
+    ga.status = ds->status;
+    ga.words_out = fin;
+    ga.words_cnt = fin_cnt;
+    ga.refine_state = state;
+    ga.refine_apair = apair;
     e = launch_gselect(ga, stream);
     if (e != cudaSuccess) return from_cuda(e);
     ds->launches += 4;
     return NEST_OK;
 }
 
-// Plan, check the scratch, launch the scan and the merge tree.  The scratch
-// (64-bit words) is the handle's own or the caller's; timing events are
-// recorded around the scan when `timed`.
-nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_t r,
+// Plan, check the scratch, launch the scan and the merge tree (or the
+// large-batch passes), then the exact re-ranking.  The scratch (64-bit
+// words) is the handle's own or the caller's; timing events are recorded
+// around the scan when `timed`.
+nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_t r_out,
                             const int64_t* seg_off, const uint32_t* key_mask, float* s_out,
                             int64_t* idx_out, uint64_t* scratch, size_t scratch_words,
                             bool timed, cudaStream_t stream)
 {
     SearchPlan sp;
-    nest_status_t st = plan_search(ds, B, r, seg_off != nullptr, &sp);
+    nest_status_t st = plan_search(ds, B, r_out, seg_off != nullptr, &sp);
     if (st != NEST_OK) return st;
     if (sp.total_words > scratch_words) return NEST_ERR_OVERFLOW;
-    uint64_t* regionA = scratch;
-    uint64_t* regionB = scratch + sp.cand_words;
-    int32_t* cntA = reinterpret_cast<int32_t*>(scratch + sp.cand_words + sp.level_words);
-    int32_t* cntB = cntA + ((size_t)sp.groups * sp.parts * sp.nq + 1) / 2 * 2;
+    const int32_t r = sp.rp;
+    uint64_t* fin = scratch + sp.off_fin;
+    int32_t* fin_cnt = reinterpret_cast<int32_t*>(fin + (size_t)B * r);
+    uint32_t* state = reinterpret_cast<uint32_t*>(fin_cnt + B);
+    auto* apair = reinterpret_cast<unsigned long long*>(fin + (size_t)B * r + (4 * (size_t)B + 1) / 2);
 
     cudaError_t e;
-    if (sp.wide)
-        return launch_wide(ds, sp, q, B, r, key_mask, s_out, idx_out, scratch, timed, stream);
-    if (sp.tc) {
-        CUtensorMap qmap;
-        if (!encode_bf16_rows(&qmap, q, B, ds->d, 16, false)) return NEST_ERR_CUDA;
-        TcScanArgs ta{};
-        ta.knorm = ds->knorm;
-        ta.q = q;
-        ta.seg_off = seg_off;
-        ta.key_mask = key_mask;
-        ta.cand = regionA;
-        ta.cand_cnt = cntA;
-        ta.status = ds->status;
-        ta.N = ds->N;
-        ta.d = ds->d;
-        ta.B = B;
-        ta.r = r;
-        ta.cap = sp.tcp.cap;
-        ta.parts = sp.tcp.parts;
-        ta.stages = sp.tcp.stages;
-        ta.kchunks = (ds->d + 63) / 64;
-        ta.key_stride = 1;
-        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
-        e = launch_tc_scan(sp.tcp, ds->keys_map, qmap, ta, stream);
+    if (sp.wide) {
+        st = launch_wide(ds, sp, q, B, key_mask, scratch, fin, fin_cnt, state, apair, timed,
+                         stream);
+        if (st != NEST_OK) return st;
     } else {
-        ScanArgs sa{};
-        sa.K = ds->K;
-        sa.knorm = ds->knorm;
-        sa.q = q;
-        sa.seg_off = seg_off;
-        sa.key_mask = key_mask;
-        sa.cand = regionA;
-        sa.cand_cnt = cntA;
-        sa.status = ds->status;
-        sa.N = ds->N;
-        sa.row_bytes = ds->row_bytes;
-        sa.chunks = ds->row_bytes / 16;
-        sa.B = B;
-        sa.r = r;
-        sa.cap = sp.scan.cap;
-        sa.parts = sp.scan.parts;
-        sa.stages = sp.scan.stages;
-        sa.stage_bytes = sp.scan.stage_bytes;
-        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
-        e = launch_scan(ds->dtype, sp.scan, sa, stream);
-    }
-    if (e != cudaSuccess) return from_cuda(e);
-    ++ds->launches;
-    if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
-
-    MergeArgs ma{};
-    ma.in = regionA;
-    ma.in_cnt = cntA;
-    ma.list_stride = (int64_t)sp.nq * r;
-    ma.nq_in = sp.nq;
-    ma.lists = sp.parts;
-    ma.B = B;
-    ma.r = r;
-    ma.s_out = s_out;
-    ma.idx_out = idx_out;
-    bool into_b = true;
-    for (;;) {
-        ma.per_cta = merge_fanin(ma.lists, r);
-        const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
-        const bool last = groups == 1;
-        ma.out = into_b ? regionB : regionA;
-        ma.out_cnt = into_b ? cntB : cntA;
-        e = launch_merge(ma, last, stream);
+        uint64_t* regionA = scratch;
+        uint64_t* regionB = scratch + sp.cand_words;
+        int32_t* cntA = reinterpret_cast<int32_t*>(scratch + sp.cand_words + sp.level_words);
+        int32_t* cntB = cntA + ((size_t)sp.groups * sp.parts * sp.nq + 1) / 2 * 2;
+        if (sp.tc) {
+            CUtensorMap qmap;
+            if (!encode_bf16_rows(&qmap, q, B, ds->d, 16, false)) return NEST_ERR_CUDA;
+            TcScanArgs ta{};
+            ta.knorm = ds->knorm;
+            ta.q = q;
+            ta.seg_off = seg_off;
+            ta.key_mask = key_mask;
+            ta.cand = regionA;
+            ta.cand_cnt = cntA;
+            ta.status = ds->status;
+            ta.N = ds->N;
+            ta.d = ds->d;
+            ta.B = B;
+            ta.r = r;
+            ta.cap = sp.tcp.cap;
+            ta.parts = sp.tcp.parts;
+            ta.stages = sp.tcp.stages;
+            ta.kchunks = (ds->d + 63) / 64;
+            ta.key_stride = 1;
+            if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+            e = launch_tc_scan(sp.tcp, ds->keys_map, qmap, ta, stream);
+        } else {
+            ScanArgs sa{};
+            sa.K = ds->K;
+            sa.knorm = ds->knorm;
+            sa.q = q;
+            sa.seg_off = seg_off;
+            sa.key_mask = key_mask;
+            sa.cand = regionA;
+            sa.cand_cnt = cntA;
+            sa.status = ds->status;
+            sa.N = ds->N;
+            sa.row_bytes = ds->row_bytes;
+            sa.chunks = ds->row_bytes / 16;
+            sa.B = B;
+            sa.r = r;
+            sa.cap = sp.scan.cap;
+            sa.parts = sp.scan.parts;
+            sa.stages = sp.scan.stages;
+            sa.stage_bytes = sp.scan.stage_bytes;
+            if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+            e = launch_scan(ds->dtype, sp.scan, sa, stream);
+        }
         if (e != cudaSuccess) return from_cuda(e);
         ++ds->launches;
-        if (last) break;
-        ma.in = ma.out;
-        ma.in_cnt = ma.out_cnt;
-        ma.list_stride = r;
-        ma.nq_in = 1;
-        ma.lists = groups;
-        into_b = !into_b;
+        if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
+
+        MergeArgs ma{};
+        ma.in = regionA;
+        ma.in_cnt = cntA;
+        ma.list_stride = (int64_t)sp.nq * r;
+        ma.nq_in = sp.nq;
+        ma.lists = sp.parts;
+        ma.B = B;
+        ma.r = r;
+        bool into_b = true;
+        for (;;) {
+            ma.per_cta = merge_fanin(ma.lists, r);
+            const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
+            const bool last = groups == 1;
+            ma.out = last ? fin : (into_b ? regionB : regionA);
+            ma.out_cnt = last ? fin_cnt : (into_b ? cntB : cntA);
+            ma.refine_state = last ? state : nullptr;
+            ma.refine_apair = last ? apair : nullptr;
+            e = launch_merge(ma, stream);
+            if (e != cudaSuccess) return from_cuda(e);
+            ++ds->launches;
+            if (last) break;
+            ma.in = ma.out;
+            ma.in_cnt = ma.out_cnt;
+            ma.list_stride = r;
+            ma.nq_in = 1;
+            ma.lists = groups;
+            into_b = !into_b;
+        }
     }
+
+    RefineArgs ra{};
+    ra.K = ds->K;
+    ra.q = q;
+    ra.row_bytes = ds->row_bytes;
+    ra.cand = fin;
+    ra.cand_cnt = fin_cnt;
+    ra.state = state;
+    ra.apair = apair;
+    ra.status = ds->status;
+    ra.B = B;
+    ra.r = sp.r;
+    ra.rp = r;
+    ra.s_out = s_out;
+    ra.idx_out = idx_out;
+    e = launch_refine(ds->dtype, ra, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+    ++ds->launches;
     return NEST_OK;
 }
 
@@ -720,6 +830,7 @@ nest_status_t nest_datastore_destroy(nest_datastore_t* ds)
     if (ds->status) keep(cudaFree(ds->status));
     if (ds->scratch) keep(cudaFree(ds->scratch));
     if (ds->host_stage) keep(cudaFree(ds->host_stage));
+    if (ds->host_status) keep(cudaFreeHost(ds->host_status));
     for (cudaEvent_t ev : ds->aux_ev)
         if (ev) keep(cudaEventDestroy(ev));
     if (ds->aux) keep(cudaStreamDestroy(ds->aux));
@@ -756,6 +867,7 @@ nest_status_t nest_knn_search(nest_datastore_t* ds, const void* q, int32_t B, in
                               const int64_t* seg_off, float* s_out, int64_t* idx_out, void* stream)
 {
     nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st == NEST_OK) st = check_device(ds);
     if (st != NEST_OK) return st;
     return run_search(ds, q, B, r, seg_off, s_out, idx_out, as_stream(stream));
 }
@@ -794,6 +906,7 @@ nest_status_t nest_knn_step(nest_datastore_t* ds, const void* q, int32_t B, int3
     st = check_mix_args(ds, s_out, idx_out, p_lm, B, r, p_knn_out, p_m_out);
     if (st != NEST_OK) return st;
     if (!(lambda >= 0.f && lambda <= 1.f)) return NEST_ERR_INVALID_ARG;
+    if ((st = check_device(ds)) != NEST_OK) return st;
     cudaStream_t s = as_stream(stream);
     st = run_search(ds, q, B, r, seg_off, s_out, idx_out, s);
     if (st != NEST_OK) return st;
@@ -854,12 +967,18 @@ nest_status_t nest_knn_step_host(nest_datastore_t* ds, const void* q, int32_t B,
     }
     st = nest_knn_mix(ds, d_s, d_i, d_p, B, r, mu, lambda, nullptr, d_m, stream);
     if (st == NEST_OK) e = cudaMemcpyAsync(p_m_out, d_m, v_bytes, cudaMemcpyDeviceToHost, s);
+    // the device status comes back with the results (and is cleared), so a
+    // condition the kernels recorded is this call's return value
+    if (st == NEST_OK && e == cudaSuccess)
+        e = cudaMemcpyAsync(ds->host_status, ds->status, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (st == NEST_OK && e == cudaSuccess) e = cudaMemsetAsync(ds->status, 0, sizeof(int), s);
     const cudaError_t es = cudaStreamSynchronize(s);
     const cudaError_t ex = cudaStreamSynchronize(x);
     if (st != NEST_OK) return st;
     if (e == cudaSuccess) e = es;
     if (e == cudaSuccess) e = ex;
-    return from_cuda(e);
+    if (e != cudaSuccess) return from_cuda(e);
+    return static_cast<nest_status_t>(*ds->host_status);
 }
 
 nest_status_t nest_knn_search_masked(nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
@@ -870,6 +989,7 @@ nest_status_t nest_knn_search_masked(nest_datastore_t* ds, const void* q, int32_
     if (st != NEST_OK) return st;
     if (!key_mask) return NEST_ERR_INVALID_ARG;
     if (!aligned(key_mask, 4)) return NEST_ERR_ALIGN;
+    if ((st = check_device(ds)) != NEST_OK) return st;
     return run_search(ds, q, B, r, seg_off, s_out, idx_out, as_stream(stream), key_mask);
 }
 
@@ -1077,6 +1197,7 @@ const char* nest_status_string(nest_status_t s)
     case NEST_ERR_OVERFLOW: return "device buffer overflow";
     case NEST_ERR_TIMEOUT: return "device wait timed out";
     case NEST_ERR_UNSUPPORTED: return "shape not supported";
+    case NEST_ERR_MARGIN: return "exact re-ranking could not confirm the r-th neighbour";
     }
     return "unknown status";
 }
@@ -1101,14 +1222,23 @@ nest_status_t search_scratch_words(const nest_datastore* ds, int32_t B, int32_t 
     return NEST_OK;
 }
 
+nest_status_t check_search_call(const nest_datastore* ds, const void* q, int32_t B, int32_t r,
+                                const int64_t* seg_off, const float* s_out,
+                                const int64_t* idx_out)
+{
+    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st == NEST_OK) st = check_device(ds);
+    return st;
+}
+
 nest_status_t search_with_scratch(nest_datastore* ds, const void* q, int32_t B, int32_t r,
                                   const int64_t* seg_off, float* s_out, int64_t* idx_out,
                                   uint64_t* scratch, size_t scratch_words, cudaStream_t stream)
 {
-    nest_status_t st = check_search_args(ds, q, B, r, seg_off, s_out, idx_out);
+    nest_status_t st = check_search_call(ds, q, B, r, seg_off, s_out, idx_out);
     if (st != NEST_OK) return st;
     return launch_search(ds, q, B, r, seg_off, nullptr, s_out, idx_out, scratch, scratch_words,
-                         false, stream);
+                         ds->timing, stream);
 }
 
 }  // namespace nest

@@ -155,16 +155,32 @@ struct WideArgs {
     // resv (one atomic per block) and pads unused slots with kNoCandidate,
     // so cnt counts reserved slots.  0: one atomic per admitting column.
     int32_t resv;
+    // Recovery pass only (launch_tc_wide_recover): per-query word limits
+    // (kNoCandidate: not recovering) and per-group flags; groups whose flag
+    // is 0 return at once.
+    const uint64_t* word_lim;
+    const int32_t* group_flag;
 };
 
 struct GselectArgs {
     uint64_t* cand;  // [B][cap]; reordered in place
-    const int32_t* cnt;
+    int32_t* cnt;    // slots taken per list (past cap when a list overflowed)
     int64_t cap;
     int32_t r;
     int32_t B;
-    float* s_out;      // B x r
+    float* s_out;      // B x r (sorted s and idx), unless words_out is set
     int64_t* idx_out;  // B x r
+    uint64_t* words_out;    // non-null: the r smallest words of each list, unsorted, [B][r]
+    int32_t* words_cnt;     // with words_out: [B] real words
+    uint32_t* refine_state;  // with words_out: the exact re-ranking's state, reset per query
+    unsigned long long* refine_apair;
+    int* status;          // with words_out: NEST_ERR_OVERFLOW if a list is still over capacity
+    // Recovery preparation (instead of any output): for an overflowed list,
+    // lim_out[q] = the r-th smallest word it holds, cnt[q] = 0 and
+    // group_flag[q / group_size] = 1; for a complete list lim_out[q] = kNoCandidate.
+    uint64_t* lim_out;
+    int32_t* group_flag;
+    int32_t group_size;
     int32_t stage_words;  // shared-memory words per CTA (set by launch_gselect)
 };
 
@@ -182,10 +198,17 @@ int wide_pair_clusters(size_t smem_limit);
 cudaError_t launch_wide_qnorm(const void* q, int32_t B, int32_t d, float* qn, cudaStream_t stream);
 cudaError_t launch_tc_wide(const WidePlan& plan, const CUtensorMap& keys,
                            const CUtensorMap& queries, const WideArgs& args, cudaStream_t stream);
+// Plan of the recovery pass for groups of nm queries: one 128-key tile per
+// stage (tc_wide_kernel), whatever kernel the main pass used.
+bool wide_recover_plan(int nm, size_t smem_limit, WidePlan* plan);
+// The recovery pass (word limits and group flags of args must be set).
+cudaError_t launch_tc_wide_recover(const WidePlan& plan, const CUtensorMap& keys,
+                                   const CUtensorMap& queries, const WideArgs& args,
+                                   cudaStream_t stream);
 cudaError_t launch_gselect(const GselectArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- merge.cu
-// Merge candidate lists of each query into its top r.
+// Merge candidate lists of each query into its r smallest words.
 struct MergeArgs {
     const uint64_t* in;    // candidate lists; list (b, l) starts at (base(b) + l * nq_in) * r with
                            // base(b) = (b / nq_in) * lists * nq_in + b % nq_in
@@ -196,17 +219,56 @@ struct MergeArgs {
     int32_t per_cta;       // lists merged by one CTA
     int32_t B;
     int32_t r;
-    uint64_t* out;         // next level: [B][ceil(lists / per_cta)][r]; unused on the last level
-    int32_t* out_cnt;      // next level: [B][ceil(lists / per_cta)]
-    float* s_out;          // last level only: B x r
-    int64_t* idx_out;      // last level only: B x r
+    uint64_t* out;         // [B][ceil(lists / per_cta)][r]
+    int32_t* out_cnt;      // [B][ceil(lists / per_cta)] real entries of each output list
+    uint32_t* refine_state;  // non-null on the final level (one list per query): the exact
+    unsigned long long* refine_apair;  // re-ranking's state is reset for each query
 };
 
 int merge_lists_per_cta(int r);
 // Lists one merge CTA takes at a level with `lists` input lists per query.
 int merge_fanin(int lists, int r);
 size_t merge_smem_bytes(int per_cta, int r);
-cudaError_t launch_merge(const MergeArgs& args, bool last, cudaStream_t stream);
+cudaError_t launch_merge(const MergeArgs& args, cudaStream_t stream);
+
+// ---------------------------------------------------------------- refine.cu
+// Exact re-ranking: each query's r' = r + refine_margin(r) screened
+// candidates get their distances recomputed as sums of squared differences;
+// the r nearest by those are sorted into s and idx.
+//
+// Per-query state: three rows of B 32-bit words (CTAs finished, largest and
+// smallest screening error as fp32 ordered bits) and B 64-bit words (the
+// largest screened distance's bits above its candidate's exact distance
+// bits).  The kernel that writes a query's candidate list resets the
+// query's entries.
+__device__ __forceinline__ void refine_state_reset(uint32_t* state, unsigned long long* apair,
+                                                   int B, int b)
+{
+    state[b] = 0;
+    state[B + b] = 0;
+    state[2 * B + b] = ~0u;
+    apair[b] = 0;
+}
+
+struct RefineArgs {
+    const void* K;
+    const void* q;       // B x d, same element type as K
+    int32_t row_bytes;   // d * element size
+    uint64_t* cand;      // [B][rp] screened words (distance bits : key), rewritten in place
+    const int32_t* cand_cnt;  // [B] real words of each list
+    uint32_t* state;     // [3][B], reset by the kernel that wrote the lists
+    unsigned long long* apair;  // [B], likewise
+    int* status;
+    int32_t B;
+    int32_t r;
+    int32_t rp;
+    float* s_out;        // B x r
+    int64_t* idx_out;    // B x r
+};
+
+int refine_margin(int r);
+size_t refine_smem_bytes(int rp, int r, int row_bytes);
+cudaError_t launch_refine(int dtype, const RefineArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- mix.cu
 struct MixArgs {
@@ -271,6 +333,11 @@ cudaError_t launch_verify(const VerifyArgs& args, cudaStream_t stream);
 cudaError_t launch_mask(uint32_t* mask, int64_t first, int64_t count, cudaStream_t stream);
 
 // ---------------------------------------------------------------- api.cu, for noalloc.cu
+// The host checks nest_knn_search makes (arguments, then the datastore's
+// device being the current one), with the same status codes.
+nest_status_t check_search_call(const nest_datastore_t* ds, const void* q, int32_t B, int32_t r,
+                                const int64_t* seg_off, const float* s_out,
+                                const int64_t* idx_out);
 // Scratch words (64-bit) a search of this shape needs; no allocation, no launch.
 nest_status_t search_scratch_words(const nest_datastore_t* ds, int32_t B, int32_t r, bool ragged,
                                    size_t* words);

@@ -1,13 +1,12 @@
-// merge.cu -- combine per-CTA candidate lists into each query's r nearest
-// neighbours (the selection of pi, Sec. 2.2 / Algorithm 1's search step).
+// merge.cu -- combine per-CTA candidate lists into each query's r' nearest
+// screened candidates (the selection of pi, Sec. 2.2 / Algorithm 1's search
+// step; refine.cu then re-ranks them by exact distance).
 //
 // A CTA copies the real entries of up to per_cta lists of one query into
 // shared memory (one warp per list, at offsets from the lists' lengths),
-// keeps the r smallest words with the same radix select the scan uses, and either writes them as one list for the next level or, on
-// the last level, sorts them (bitonic) and writes s = -distance and the key
-// index, nearest first, ties by smaller index, padding with (-inf, -1).
-#include <cmath>
-
+// keeps the r' smallest words with the same radix select the scan uses, and
+// writes them as one list: for the next level, or, on the final level (one
+// CTA per query), for the exact re-ranking.
 #include "internal.h"
 #include "ptx.cuh"
 #include "select.cuh"
@@ -40,7 +39,6 @@ __host__ __device__ inline size_t buf_words(int per_cta, int r)
     return a > b ? a : b;
 }
 
-template <bool LAST>
 __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
@@ -103,27 +101,13 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
                                       [] { __syncthreads(); });
     const int n = sh.cnt;
 
-    if constexpr (!LAST) {
-        uint64_t* dst = a.out + ((int64_t)b * gridDim.x + grp) * a.r;
-        for (int j = tid; j < a.r; j += kMergeThreads) dst[j] = j < n ? buf[j] : kNoCandidate;
-        if (tid == 0) a.out_cnt[(int64_t)b * gridDim.x + grp] = n;
-    } else {
-        const int P2 = next_pow2(n > 0 ? n : 1);
-        for (int j = n + tid; j < P2; j += kMergeThreads) buf[j] = kNoCandidate;
-        __syncthreads();
-        bitonic_sort<kMergeThreads>(buf, P2, tid, [] { __syncthreads(); });
-        float* so = a.s_out + (int64_t)b * a.r;
-        int64_t* io = a.idx_out + (int64_t)b * a.r;
-        for (int j = tid; j < a.r; j += kMergeThreads) {
-            if (j < n) {
-                const uint64_t e = buf[j];
-                so[j] = -__uint_as_float((uint32_t)(e >> 32));
-                io[j] = (int64_t)(uint32_t)e;
-            } else {
-                so[j] = -INFINITY;
-                io[j] = -1;
-            }
-        }
+    uint64_t* dst = a.out + ((int64_t)b * gridDim.x + grp) * a.r;
+    for (int j = tid; j < a.r; j += kMergeThreads) dst[j] = j < n ? buf[j] : kNoCandidate;
+    if (tid == 0) {
+        a.out_cnt[(int64_t)b * gridDim.x + grp] = n;
+        // the final level hands the query's list to the exact re-ranking
+        if (a.refine_state != nullptr)
+            refine_state_reset(a.refine_state, a.refine_apair, a.B, b);
     }
 }
 
@@ -154,21 +138,14 @@ size_t merge_smem_bytes(int per_cta, int r)
     return buf_words(per_cta, r) * 8 + sizeof(MergeShared);
 }
 
-cudaError_t launch_merge(const MergeArgs& a, bool last, cudaStream_t stream)
+cudaError_t launch_merge(const MergeArgs& a, cudaStream_t stream)
 {
     const int groups = (a.lists + a.per_cta - 1) / a.per_cta;
     const size_t smem = merge_smem_bytes(a.per_cta, a.r);
     const dim3 grid(groups, a.B);
-    cudaError_t e;
-    if (last) {
-        e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel<true>), (int)smem);
-        if (e != cudaSuccess) return e;
-        merge_kernel<true><<<grid, kMergeThreads, smem, stream>>>(a);
-    } else {
-        e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel<false>), (int)smem);
-        if (e != cudaSuccess) return e;
-        merge_kernel<false><<<grid, kMergeThreads, smem, stream>>>(a);
-    }
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel), (int)smem);
+    if (e != cudaSuccess) return e;
+    merge_kernel<<<grid, kMergeThreads, smem, stream>>>(a);
     return cudaGetLastError();
 }
 

@@ -59,10 +59,11 @@ extern "C" nest_status_t nest_knn_search_static(nest_datastore_t* ds, const void
                                                 int32_t r, const int64_t* seg_off, float* s_out,
                                                 int64_t* idx_out, void* stream)
 {
-    if (!ds || !q || !s_out || !idx_out) return NEST_ERR_INVALID_ARG;
-    if (B < 1 || r < 1 || r > NEST_MAX_R) return NEST_ERR_INVALID_ARG;
+    // the argument, alignment and device checks of nest_knn_search come first
+    nest_status_t st = nest::check_search_call(ds, q, B, r, seg_off, s_out, idx_out);
+    if (st != NEST_OK) return st;
     size_t need = 0;
-    nest_status_t st = nest::search_scratch_words(ds, B, r, seg_off != nullptr, &need);
+    st = nest::search_scratch_words(ds, B, r, seg_off != nullptr, &need);
     if (st != NEST_OK) return st;
     if (need > kStaticScratchWords) return NEST_ERR_OVERFLOW;
     uint64_t* scratch = nullptr;

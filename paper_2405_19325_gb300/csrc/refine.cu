@@ -1,0 +1,246 @@
+// refine.cu -- exact re-ranking of each query's screened candidates (the
+// r nearest keys by s(q, k) = -||q - k||^2, Sec. 2.2 / App. A).
+//
+// The scans rank keys by ||q||^2 + ||k||^2 - 2 q.k evaluated in fp32.  Its
+// rounding error is absolute in the norms (the dot product is accumulated
+// over d terms of the size of ||q|| ||k||), so two keys whose distances
+// differ by less than that error can come out in either order, and a key
+// very close to the query gets a distance with a large relative error.  The
+// searches therefore keep r' = r + margin candidates per query, and this
+// kernel recomputes each candidate's distance directly as the sum of the
+// squared differences of the stored elements (fp32, exact products of the
+// widened bf16 values; eight interleaved partial sums per lane and a warp
+// tree, so at most ~40 additions separate any term from the result).  It
+// then keeps the r nearest by those distances (ties: smaller key index),
+// sorts them and writes s = -distance and the key index.
+//
+// Grid (chunks of 32 candidates, B queries), 1024 threads: warp w of chunk c
+// recomputes candidate 32 c + w.  A CTA rewrites its candidates' words in
+// place, and the last CTA of a query to finish (an atomic counter, no wait)
+// selects, sorts and writes the row.
+//
+// It also checks the margin.  A key left out of the r' candidates had a
+// screened distance of at least A, the largest screened distance kept.  The
+// screening errors e = screened - exact of the candidates span [e_min, e_max]
+// (mostly a common offset: the accumulation error grows with ||q|| ||k||,
+// which is about the same for keys at about the same distance).  Taking an
+// excluded key's error to exceed that of the candidate at A by at most
+// W = 2 (e_max - e_min), its exact distance is at least A_exact - W, where
+// A_exact is the exact distance of that candidate.  So the r nearest are
+// certain when A_exact - W > D_r, the r-th exact distance.  When instead the
+// candidate at A ties the r-th exactly, the boundary lies inside a run of
+// exact ties (duplicated keys: equal screened and exact distances, broken
+// by index the same way in both), which also passes.  Otherwise a key
+// outside the candidates might belong to the r nearest and NEST_ERR_MARGIN
+// is recorded.
+#include <cmath>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "select.cuh"
+
+namespace nest {
+namespace {
+
+constexpr int kRefineThreads = 1024;
+constexpr int kRefineRows = kRefineThreads / 32;  // candidates per CTA
+// Distance bits no real distance has (a NaN pattern above +inf's bits).
+constexpr uint64_t kPadHigh = 0xFFFFFFFFull << 32;
+
+// fp32 values as unsigned integers that order like the values.
+__device__ __forceinline__ uint32_t ordered_bits(float x)
+{
+    const uint32_t u = __float_as_uint(x);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float from_ordered_bits(uint32_t o)
+{
+    return __uint_as_float((o & 0x80000000u) ? (o & 0x7fffffffu) : ~o);
+}
+
+struct RefineShared {
+    uint32_t emax, emin;      // largest / smallest screened - exact distance (ordered bits)
+    unsigned long long apair; // largest (screened bits << 32 | exact bits) of this CTA
+    int last;
+    int cnt;
+    uint64_t thr;
+    SelectSmem<kRefineThreads, 1> sel;
+};
+
+__host__ __device__ inline int pow2_at_least(int x)
+{
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+// Sum of squared differences of one 16-byte chunk (8 bf16 or 4 fp32 values)
+// into the lane's partial sums.
+template <int DT>
+__device__ __forceinline__ void chunk_sqdiff(const uint4& k, const uint4& q, float (&acc)[8])
+{
+    const uint32_t kw[4] = {k.x, k.y, k.z, k.w};
+    const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+    if constexpr (DT == NEST_BF16) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float d0 = __uint_as_float(qw[i] << 16) - __uint_as_float(kw[i] << 16);
+            const float d1 = __uint_as_float(qw[i] & 0xffff0000u) - __uint_as_float(kw[i] & 0xffff0000u);
+            acc[2 * i] = fmaf(d0, d0, acc[2 * i]);
+            acc[2 * i + 1] = fmaf(d1, d1, acc[2 * i + 1]);
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float d0 = __uint_as_float(qw[i]) - __uint_as_float(kw[i]);
+            acc[i] = fmaf(d0, d0, acc[i]);
+        }
+    }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kRefineThreads, 1) refine_kernel(const RefineArgs a)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint4* qs = reinterpret_cast<uint4*>(smem);  // the query row
+    uint64_t* buf = reinterpret_cast<uint64_t*>(smem + a.row_bytes);
+    __shared__ RefineShared sh;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int b = blockIdx.y;
+    const int chunks = a.row_bytes / 16;
+    uint64_t* list = a.cand + (int64_t)b * a.rp;
+    const int n = min(max(a.cand_cnt[b], 0), a.rp);
+
+    const uint4* qrow = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(a.q) +
+                                                       (size_t)b * a.row_bytes);
+    for (int c = tid; c < chunks; c += kRefineThreads) qs[c] = ld_global_nc_v4(qrow + c);
+    if (tid == 0) {
+        sh.emax = 0;
+        sh.emin = ~0u;
+        sh.apair = 0;
+    }
+    __syncthreads();
+
+    // ---- one warp per candidate: exact distance, word rewritten in place
+    const int j = blockIdx.x * kRefineRows + warp;
+    if (j < n) {
+        const uint64_t w = list[j];
+        if (w != kNoCandidate) {
+            const uint32_t key = (uint32_t)w;
+            const uint4* krow = reinterpret_cast<const uint4*>(
+                static_cast<const unsigned char*>(a.K) + (size_t)key * a.row_bytes);
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            int c = lane;
+            for (; c + 3 * 32 < chunks; c += 4 * 32) {
+                uint4 kv[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) kv[u] = ld_global_nc_v4(krow + c + 32 * u);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) chunk_sqdiff<DT>(kv[u], qs[c + 32 * u], acc);
+            }
+            for (; c < chunks; c += 32) chunk_sqdiff<DT>(ld_global_nc_v4(krow + c), qs[c], acc);
+            float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
+            if (lane == 0) {
+                const float screened = __uint_as_float((uint32_t)(w >> 32));
+                list[j] = ((uint64_t)__float_as_uint(s) << 32) | key;
+                __threadfence();  // the word is visible before this CTA counts itself done
+                const uint32_t e = ordered_bits(screened - s);
+                atomicMax(&sh.emax, e);
+                atomicMin(&sh.emin, e);
+                // distances are >= 0, so their bits order like the values
+                atomicMax(&sh.apair, ((unsigned long long)(w >> 32) << 32) | __float_as_uint(s));
+            }
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        atomicMax(&a.state[a.B + b], sh.emax);
+        atomicMin(&a.state[2 * a.B + b], sh.emin);
+        atomicMax(&a.apair[b], sh.apair);
+        __threadfence();
+        const uint32_t prev = atomicAdd(&a.state[b], 1u);
+        sh.last = prev == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!sh.last) return;
+    __threadfence();
+
+    // ---- last CTA of this query: r nearest by exact distance, sorted.  A
+    // padding word (none is expected among the n) becomes a distinct word
+    // above every real one, so the select sees distinct words.
+    for (int i = tid; i < n; i += kRefineThreads) {
+        const uint64_t w = __ldcg(list + i);
+        buf[i] = w != kNoCandidate ? w : (kPadHigh | (uint32_t)i);
+    }
+    if (tid == 0) {
+        sh.cnt = n;
+        sh.thr = kNoCandidate;
+    }
+    __syncthreads();
+    select_smallest<kRefineThreads, 1>(buf, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
+                                       [] { __syncthreads(); });
+    const int m = sh.cnt;
+    const int P2 = pow2_at_least(m > 0 ? m : 1);
+    for (int i = m + tid; i < P2; i += kRefineThreads) buf[i] = kNoCandidate;
+    __syncthreads();
+    bitonic_sort<kRefineThreads>(buf, P2, tid, [] { __syncthreads(); });
+    float* so = a.s_out + (int64_t)b * a.r;
+    int64_t* io = a.idx_out + (int64_t)b * a.r;
+    for (int i = tid; i < a.r; i += kRefineThreads) {
+        const uint64_t e = i < m ? buf[i] : kNoCandidate;
+        if ((e >> 32) != 0xFFFFFFFFu) {
+            so[i] = -__uint_as_float((uint32_t)(e >> 32));
+            io[i] = (int64_t)(uint32_t)e;
+        } else {
+            so[i] = -INFINITY;
+            io[i] = -1;
+        }
+    }
+    if (tid == 0) {
+        // Keys outside the candidates exist only when the list is full.
+        if (n == a.rp && m == a.r) {
+            const float A_exact = __uint_as_float((uint32_t)__ldcg(&a.apair[b]));
+            const float emax = from_ordered_bits(__ldcg(&a.state[a.B + b]));
+            const float emin = from_ordered_bits(__ldcg(&a.state[2 * a.B + b]));
+            const float Dr = __uint_as_float((uint32_t)(buf[a.r - 1] >> 32));
+            const float W = 2.f * (emax - emin);
+            const bool ok = (A_exact - W > Dr) || (A_exact == Dr);
+            if (!ok) record_status(a.status, NEST_ERR_MARGIN);
+        }
+        // ready for the next search (the kernel before this one also resets them)
+        refine_state_reset(a.state, a.apair, a.B, b);
+    }
+}
+
+}  // namespace
+
+int refine_margin(int r)
+{
+    const int m = r / 16;
+    return m < 16 ? 16 : (m > 128 ? 128 : m);
+}
+
+size_t refine_smem_bytes(int rp, int r, int row_bytes)
+{
+    const int words = rp > pow2_at_least(r) ? rp : pow2_at_least(r);
+    return (size_t)row_bytes + (size_t)words * sizeof(uint64_t);
+}
+
+cudaError_t launch_refine(int dtype, const RefineArgs& a, cudaStream_t stream)
+{
+    const dim3 grid((a.rp + kRefineRows - 1) / kRefineRows, a.B);
+    const size_t smem = refine_smem_bytes(a.rp, a.r, a.row_bytes);
+    const void* kern = dtype == NEST_BF16 ? reinterpret_cast<const void*>(refine_kernel<NEST_BF16>)
+                                          : reinterpret_cast<const void*>(refine_kernel<NEST_F32>);
+    cudaError_t e = raise_smem_limit(kern, smem);
+    if (e != cudaSuccess) return e;
+    if (dtype == NEST_BF16)
+        refine_kernel<NEST_BF16><<<grid, kRefineThreads, smem, stream>>>(a);
+    else
+        refine_kernel<NEST_F32><<<grid, kRefineThreads, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace nest

@@ -85,11 +85,13 @@ __device__ __forceinline__ void wait_or_abort_w(uint64_t* bar, uint32_t parity, 
 }
 
 // Pads slots [from, to) of list `col` with kNoCandidate (reserved, never written).
+// Slot numbers are taken as unsigned: a count that has passed 2^31 (far
+// beyond any list) writes nothing.
 __device__ __forceinline__ void wide_pad(const WideArgs& a, int64_t col, int from, int to)
 {
     uint64_t* list = a.cand + col * a.cap;
-    const int end = to < a.cap ? to : (int)a.cap;
-    for (int p = from; p < end; ++p) list[p] = kNoCandidate;
+    const uint64_t end = (uint32_t)to < (uint64_t)a.cap ? (uint32_t)to : (uint64_t)a.cap;
+    for (uint64_t p = (uint32_t)from; p < end; ++p) list[p] = kNoCandidate;
 }
 
 // Epilogue of W accumulator columns (queries c0 .. c0 + W - 1) of one key
@@ -108,12 +110,32 @@ __device__ __forceinline__ void wide_pad(const WideArgs& a, int64_t col, int fro
 //    column i's list (from the warp's block, or with one global atomic; all
 //    columns' atomics in flight together), and every admitting lane writes
 //    its word.
-template <int W, int NM>
+template <int W, int NM, bool WORD = false>
 __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, int nqv, float kn,
                                              bool valid, uint32_t key_idx, int64_t pos, int lane,
                                              const WideShared<NM>& sh, int2* resv,
                                              uint32_t* stage, const WideArgs& a, int q0)
 {
+    if constexpr (WORD) {
+        // Recovery pass of overflowed lists: a key is admitted when its whole
+        // word (distance bits, key index) is at or below the query's limit
+        // (kNoCandidate: the query is not recovering), one list slot per key.
+        if (!valid) return;
+#pragma unroll 1
+        for (int i = 0; i < W; ++i) {
+            const int col = c0 + i;
+            if (col >= nqv) break;
+            const uint64_t lim = __ldg(a.word_lim + q0 + col);
+            float dist = fmaf(-2.f, __uint_as_float(acc[i]), sh.qn[col] + kn);
+            dist = (dist <= 0.f) ? 0.f : dist;
+            const uint64_t w = ((uint64_t)__float_as_uint(dist) << 32) | key_idx;
+            if (lim != kNoCandidate && w <= lim) {
+                const uint32_t slot = (uint32_t)atomicAdd(&a.cnt[q0 + col], 1);
+                if (slot < (uint64_t)a.cap) a.cand[(int64_t)(q0 + col) * a.cap + slot] = w;
+            }
+        }
+        return;
+    }
     if (a.s_sample == nullptr) {
         // every key is admitted: the word of tensor-map row `pos` goes to
         // position `pos` of each list (masked keys leave a padding word)
@@ -186,10 +208,10 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
             dbits = (int)dbits < 0 ? 0u : dbits;  // D <= 0 is stored as 0
             int slot = atomicAdd(&resv[col].x, 1);
             if (slot >= resv[col].y) slot = atomicAdd(&a.cnt[q0 + col], 1);
-            if (slot < a.cap)
+            // a full list drops the key; its count keeps growing past the
+            // capacity, which the selection after the pass detects
+            if ((uint32_t)slot < (uint64_t)a.cap)
                 a.cand[(int64_t)(q0 + col) * a.cap + slot] = ((uint64_t)dbits << 32) | key_idx;
-            else
-                record_status(a.status, NEST_ERR_OVERFLOW);
         }
         __syncwarp();
         return;
@@ -232,9 +254,8 @@ __device__ __forceinline__ void wide_columns(const uint32_t (&acc)[W], int c0, i
             float dist = fmaf(-2.f, __uint_as_float(acc[i]), sh.qn[c0 + i] + kn);
             dist = (dist <= 0.f) ? 0.f : dist;
             const uint64_t key = ((uint64_t)__float_as_uint(dist) << 32) | key_idx;
-            const long long pos = (long long)at + __popc(bal & lt);
-            if (pos < a.cap) a.cand[(int64_t)(q0 + c0 + i) * a.cap + pos] = key;
-            else record_status(a.status, NEST_ERR_OVERFLOW);
+            const uint64_t pos = (uint64_t)(uint32_t)at + __popc(bal & lt);
+            if (pos < (uint64_t)a.cap) a.cand[(int64_t)(q0 + c0 + i) * a.cap + pos] = key;
         }
     }
 }
@@ -275,7 +296,7 @@ __device__ __forceinline__ void wide_release(const int2* resv, int c_begin, int 
 // the next load is in flight while the current columns are tested (more
 // registers); without it the other warps of the SM sub-partition hide the
 // load latency.
-template <int NM, int NCOL, bool PIPE, bool CLUSTER_RELEASE = false>
+template <int NM, int NCOL, bool PIPE, bool CLUSTER_RELEASE = false, bool WORD = false>
 __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint64_t* release,
                                                int nqv, float kn, bool valid, uint32_t key_idx,
                                                int64_t pos, int lane, const WideShared<NM>& sh,
@@ -296,8 +317,8 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
             tmem_ld_32_async(tbase + (uint32_t)c0, acc);
             tmem_wait_ld(acc);
             if (c0 + 32 == NCOL) hand_back();
-            wide_columns<32, NM>(acc, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage,
-                                 a, q0);
+            wide_columns<32, NM, WORD>(acc, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh,
+                                       resv, stage, a, q0);
         }
         return;
     }
@@ -311,8 +332,8 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
         } else {
             hand_back();
         }
-        wide_columns<32, NM>(a0, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage, a,
-                             q0);
+        wide_columns<32, NM, WORD>(a0, c_base + c0, nqv, kn, valid, key_idx, pos, lane, sh, resv,
+                                   stage, a, q0);
         if (c0 + 32 < NCOL) {
             tmem_wait_ld(a1);
             if (c0 + 64 < NCOL) {
@@ -320,13 +341,13 @@ __device__ __forceinline__ void wide_drain_row(uint32_t tbase, int c_base, uint6
             } else {
                 hand_back();
             }
-            wide_columns<32, NM>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, pos, lane, sh, resv,
-                                 stage, a, q0);
+            wide_columns<32, NM, WORD>(a1, c_base + c0 + 32, nqv, kn, valid, key_idx, pos, lane, sh,
+                                       resv, stage, a, q0);
         }
     }
 }
 
-template <int NM>
+template <int NM, bool WORD = false>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_wide_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
                    const WideArgs a)
@@ -348,6 +369,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int part = blockIdx.x / a.groups, group = blockIdx.x - part * a.groups;
     const int q0 = group * NM;
     const int nqv = min(NM, a.B - q0);
+    // a recovery pass runs only for groups with an overflowed list
+    if constexpr (WORD) {
+        if (a.group_flag[group] == 0) return;
+    }
 
     const int64_t tiles = (a.N + kTileM - 1) / kTileM;
     const int64_t t0 = tiles * part / a.parts, t1 = tiles * (part + 1) / a.parts;
@@ -488,10 +513,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tmem_ld_16(tbase, acc);
                 tc_fence_before();
                 mbar_arrive(&sh.acc_empty[buf]);
-                wide_columns<16, NM>(acc, 0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage, a, q0);
+                wide_columns<16, NM, WORD>(acc, 0, nqv, kn, valid, key_idx, pos, lane, sh, resv, stage,
+                                           a, q0);
             } else {
-                wide_drain_row<NM, NM, true>(tbase, 0, &sh.acc_empty[buf], nqv, kn, valid, key_idx, pos, lane,
-                                       sh, resv, stage, a, q0);
+                wide_drain_row<NM, NM, true, false, WORD>(tbase, 0, &sh.acc_empty[buf], nqv, kn, valid,
+                                                          key_idx, pos, lane, sh, resv, stage, a, q0);
             }
         }
         wide_release(resv, 0, NM, nqv, lane, a, q0);
@@ -978,8 +1004,17 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int q = blockIdx.x;
     uint64_t* list = a.cand + (int64_t)q * a.cap;
-    const int c = a.cnt[q];
-    const int n = c < a.cap ? c : (int)a.cap;
+    // slots taken, which keep counting past the capacity when a list overflows
+    const uint32_t c = (uint32_t)a.cnt[q];
+    const bool overflowed = c > (uint64_t)a.cap;
+    const int n = overflowed ? (int)a.cap : (int)c;
+    if (a.lim_out != nullptr && !overflowed) {
+        // recovery preparation: this list is complete, nothing to redo
+        if (threadIdx.x == 0) a.lim_out[q] = kNoCandidate;
+        return;
+    }
+    if (a.words_out != nullptr && overflowed && threadIdx.x == 0)
+        record_status(a.status, NEST_ERR_OVERFLOW);  // recovery did not bring it under the capacity
     if (tid == 0) {
         sh.hmin = ~0u;
         sh.hmax = 0;
@@ -1087,6 +1122,34 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
                                         [] { __syncthreads(); });
         nsel = sh.cnt;
         for (int j = tid; j < nsel; j += kSelThreads) stage[j] = list[j];
+    }
+    if (a.lim_out != nullptr) {
+        // Recovery preparation of an overflowed list: the r-th smallest of
+        // the words it holds bounds the r-th smallest of all keys from
+        // above, so a pass admitting every word up to it misses none of the
+        // r nearest.  The list starts over; its group is flagged.
+        __shared__ unsigned long long lim;
+        if (tid == 0) lim = 0;
+        __syncthreads();
+        for (int j = tid; j < nsel; j += kSelThreads)
+            if (stage[j] != kNoCandidate) atomicMax(&lim, (unsigned long long)stage[j]);
+        __syncthreads();
+        if (tid == 0) {
+            a.lim_out[q] = lim;
+            a.cnt[q] = 0;
+            a.group_flag[q / a.group_size] = 1;
+        }
+        return;
+    }
+    if (a.words_out != nullptr) {
+        // the r smallest words, unsorted, for the exact re-ranking
+        uint64_t* wo = a.words_out + (int64_t)q * a.r;
+        for (int j = tid; j < a.r; j += kSelThreads) wo[j] = j < nsel ? stage[j] : kNoCandidate;
+        if (tid == 0) {
+            a.words_cnt[q] = nsel;
+            refine_state_reset(a.refine_state, a.refine_apair, a.B, q);
+        }
+        return;
     }
     int P2 = 1;
     while (P2 < (nsel > 0 ? nsel : 1)) P2 <<= 1;
@@ -1212,6 +1275,62 @@ int wide_pair_clusters(size_t smem_limit)
         return 0;
     }
     return n;
+}
+
+namespace {
+
+template <int NM>
+bool wide_recover_plan_nm(size_t smem_limit, WidePlan* p)
+{
+    const size_t fixed = wide_fixed<NM>();
+    const size_t st = (size_t)stage_bytes<NM>();
+    if (fixed + 3 * st > smem_limit) return false;
+    int stages = (int)((smem_limit - fixed) / st);
+    stages = stages > kMaxStagesW ? kMaxStagesW : stages;
+    p->nm = NM;
+    p->mb = 1;
+    p->pair = false;
+    p->stages = stages;
+    p->smem = fixed + (size_t)stages * st;
+    return true;
+}
+
+template <int NM>
+cudaError_t recover_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
+                              const WideArgs& a, cudaStream_t stream)
+{
+    auto kern = tc_wide_kernel<NM, true>;
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
+    if (e != cudaSuccess) return e;
+    kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool wide_recover_plan(int nm, size_t smem_limit, WidePlan* p)
+{
+    switch (nm) {
+    case 16: return wide_recover_plan_nm<16>(smem_limit, p);
+    case 32: return wide_recover_plan_nm<32>(smem_limit, p);
+    case 64: return wide_recover_plan_nm<64>(smem_limit, p);
+    case 128: return wide_recover_plan_nm<128>(smem_limit, p);
+    case 256: return wide_recover_plan_nm<256>(smem_limit, p);
+    default: return false;
+    }
+}
+
+cudaError_t launch_tc_wide_recover(const WidePlan& p, const CUtensorMap& tmK,
+                                   const CUtensorMap& tmQ, const WideArgs& a, cudaStream_t stream)
+{
+    switch (p.nm) {
+    case 16: return recover_launch_nm<16>(p, tmK, tmQ, a, stream);
+    case 32: return recover_launch_nm<32>(p, tmK, tmQ, a, stream);
+    case 64: return recover_launch_nm<64>(p, tmK, tmQ, a, stream);
+    case 128: return recover_launch_nm<128>(p, tmK, tmQ, a, stream);
+    case 256: return recover_launch_nm<256>(p, tmK, tmQ, a, stream);
+    default: return cudaErrorInvalidValue;
+    }
 }
 
 cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,

@@ -21,7 +21,7 @@ BF16 = 1
 STATUS = {
     0: "NEST_OK", 1: "NEST_ERR_INVALID_ARG", 2: "NEST_ERR_DTYPE", 3: "NEST_ERR_ALIGN",
     4: "NEST_ERR_OOM", 5: "NEST_ERR_CUDA", 6: "NEST_ERR_VALUE_RANGE", 7: "NEST_ERR_OVERFLOW",
-    8: "NEST_ERR_TIMEOUT", 9: "NEST_ERR_UNSUPPORTED",
+    8: "NEST_ERR_TIMEOUT", 9: "NEST_ERR_UNSUPPORTED", 10: "NEST_ERR_MARGIN",
 }
 STATUS_CODE = {v: k for k, v in STATUS.items()}
 

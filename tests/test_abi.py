@@ -79,6 +79,12 @@ def test_search_and_mix_validation(lib):
     assert lib.nest_knn_search(ds, P(FAKE + 8), 1, 1, None, s, i, None) == 3
     assert lib.nest_knn_search(ds, q, 1, 1, P(FAKE + 4), s, i, None) == 3
     assert lib.nest_knn_search(ds, q, 1, 1, None, s, P(FAKE + 4), None) == 3
+    # the allocation-free search makes the same checks first, before its size check
+    assert lib.nest_knn_search_static(None, q, 1, 1, None, s, i, None) == 1
+    assert lib.nest_knn_search_static(ds, q, 65536, 1, None, s, i, None) == 1
+    assert lib.nest_knn_search_static(ds, q, 1, 4097, None, s, i, None) == 1
+    assert lib.nest_knn_search_static(ds, P(FAKE + 8), 1, 1, None, s, i, None) == 3
+    assert lib.nest_knn_search_static(ds, q, 1, 1, P(FAKE + 4), s, i, None) == 3
     p = P(FAKE)
     assert lib.nest_knn_mix(ds, s, i, p, 1, 1, 1.0, 1.5, None, p, None) == 1
     assert lib.nest_knn_mix(ds, s, i, p, 1, 1, 1.0, -0.1, None, p, None) == 1

@@ -38,7 +38,7 @@ def _cand_counts(B, N, seg_off):
 
 
 def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, exact=False,
-                  oracle_threads=None, check_rows=None, pairs=None):
+                  oracle_threads=None, check_rows=None, pairs=None, label=None):
     """GPU step through the C ABI, then the oracle on the same bytes.
 
     ``check_rows`` restricts the oracle (and the comparison) to those query
@@ -64,7 +64,8 @@ def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, e
     ref = oracle.knn_step(K_np, V_np, q_np, r, p_lm_np, mu, lam, vocab, seg_off=so_np,
                           nthreads=oracle_threads)
     rows = check_search(s_g, i_g, ref["s"], ref["idx"], K_np, q_np, dtype,
-                        _cand_counts(q_np.shape[0], K.shape[0], seg_off), exact=exact)
+                        _cand_counts(q_np.shape[0], K.shape[0], seg_off), exact=exact,
+                        label=label)
     p_m = out["p_m"].cpu().numpy()[rows_sel]
     check_mix(p_m, s_g, i_g, V_np, p_lm_np, mu, lam, vocab,
               p_knn_gpu=out["p_knn"].cpu().numpy()[rows_sel])
@@ -78,7 +79,8 @@ def run_and_check(nest, K, V, q, p_lm, r, mu, lam, vocab, dtype, seg_off=None, e
 def test_tiny_workload(nest):
     w = synth.WORKLOADS["tiny"]
     x = synth.make_inputs(w)
-    _, _, rows = run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype)
+    _, _, rows = run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
+                               label="config 1: tiny fp32 d=64")
     assert len(rows) == w.B
 
 
@@ -86,7 +88,8 @@ def test_decode_workload_full_size(nest):
     """bf16 d=4096, N=1,048,576 clustered keys, B=4, r=1024: the benchmarked launch."""
     w = synth.WORKLOADS["decode"]
     x = synth.make_inputs(w, device="cuda")
-    run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype)
+    run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
+                  label="config 2: decode, 1M keys, d=4096, r=1024")
 
 
 def test_ragged_workload_full_size(nest):
@@ -94,7 +97,7 @@ def test_ragged_workload_full_size(nest):
     w = synth.WORKLOADS["ragged"]
     x = synth.make_inputs(w, device="cuda")
     _, _, rows = run_and_check(nest, x.K, x.V, x.q, x.p_lm, w.r, w.mu, w.lam, w.vocab, w.dtype,
-                               seg_off=x.seg_off)
+                               seg_off=x.seg_off, label="config 3: ragged, 32 x 10,240 keys")
     assert len(rows) >= w.B // 2
 
 
@@ -162,6 +165,47 @@ def test_key_equal_to_query_is_first_with_distance_zero(nest):
     p_lm = torch.softmax(torch.randn(3, 100, generator=g), dim=1)
     out, _, _ = run_and_check(nest, K, V, q, p_lm, 10, 1 / np.sqrt(128), 0.8, 100, "bf16")
     assert out["idx"][:, 0].cpu().tolist() == [17, 9999, 4242]
+
+
+def test_margin_check_reports_a_crowded_boundary(nest):
+    """Keys whose exact distances are packed closer than the fp32 screening
+    error: integer vectors of about 1,000-norm-squared per element (||q||^2 and
+    ||k||^2 near 3.7e7, so ||q||^2 + ||k||^2 - 2 q.k carries errors of several
+    units), each the query plus a and b in two positions (a, b < 16), so
+    D = a^2 + b^2 exactly.  Hundreds of keys lie within the screening error of
+    the 16th distance, far more than the 16 extra candidates the re-ranking
+    keeps.  The search must either return the oracle's neighbours or report
+    NEST_ERR_MARGIN; on this data it reports it."""
+    g = torch.Generator().manual_seed(77)
+    d, N, r = 1024, 4096, 16
+    c = torch.randint(128, 256, (d,), generator=g).float()
+    K = c.repeat(N, 1)
+    i = torch.arange(N)
+    a = torch.randint(0, 16, (N,), generator=g).float()
+    b = torch.randint(0, 16, (N,), generator=g).float()
+    K[i, i % 1000] += a
+    K[i, (7 * i + 3) % 1000 + 1] += b
+    K = K.to(torch.bfloat16)
+    assert torch.equal(K.float(), K.float().round())  # integers, exact in bf16
+    q = c.to(torch.bfloat16).repeat(2, 1)
+    V = torch.randint(0, 10, (N,), generator=g, dtype=torch.int32)
+    ds = nest.Datastore(K.cuda(), V.cuda(), 10)
+    s, idx = ds.search(q.cuda(), r)
+    torch.cuda.synchronize()
+    st = ds.device_status()
+    ds.close()
+    K_np, q_np = _np(K), _np(q)
+    s_or, i_or = oracle.knn_search(K_np, q_np, r)
+    if st == 0:
+        check_search(s.cpu().numpy(), idx.cpu().numpy(), s_or, i_or, K_np, q_np, "bf16",
+                     np.full(2, N), exact=True)
+    else:
+        assert st == nest.nest.STATUS_CODE["NEST_ERR_MARGIN"]
+        # the rows still hold r distinct keys with exact distances, nearest first
+        D = -s.cpu().double().numpy()
+        D_ex = oracle.sqdist(K_np[idx.cpu().numpy()[0]], q_np[:1])[0]
+        assert np.array_equal(D[0], D_ex) and np.all(np.diff(D[0]) >= 0)
+    assert st == nest.nest.STATUS_CODE["NEST_ERR_MARGIN"], "expected the crowded boundary flagged"
 
 
 def test_ragged_edges(nest):
@@ -458,6 +502,41 @@ def test_wide_batch_massive_exact_ties(nest, pairs):
                   pairs=pairs)
 
 
+@pytest.mark.parametrize("B", [40, 300])
+def test_wide_batch_list_overflow_is_recovered(nest, B):
+    """50,000 exact copies of one vector among 200,000 keys, and queries next
+    to it: the sample's r-th distance is the copies' distance, so the
+    thresholded pass admits every copy, far more than a query's list holds.
+    The overflowed lists are scanned again with the r-th smallest word each
+    holds as the limit (ties broken by key index), and the search returns the
+    oracle's exact neighbours -- the copies with the smallest indices -- with
+    no error.  B = 40 runs the groups-of-64 kernel, B = 300 the groups-of-256
+    one; bf16, d=64, r=16."""
+    g = torch.Generator().manual_seed(91)
+    N, d, r, vocab, n_copies = 200000, 64, 16, 300, 50000
+    K = torch.randn(N, d, generator=g)
+    v = torch.randn(d, generator=g)
+    pos = torch.randperm(N, generator=g)[:n_copies]
+    K[pos] = v
+    K = K.to(torch.bfloat16)
+    q = torch.randn(B, d, generator=g)
+    near = torch.arange(0, B, 2)
+    q[near] = v + 0.05 * torch.randn(len(near), d, generator=g)
+    q = q.to(torch.bfloat16)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g), dim=1)
+    plan = nest.plan_offline(N, d, "bf16", B, r)
+    assert plan["path"] in (2, 3) and not plan["single_pass"]
+    assert plan["list_capacity"] < n_copies  # every copy is admitted: the lists overflow
+    rows = sorted(set(list(range(0, B, max(1, B // 12))) + [1, B - 1, B - 2]))
+    out, ref, exact_rows = run_and_check(nest, K, V, q, p_lm, r, 1 / 8, 0.7, vocab, "bf16",
+                                         check_rows=rows)
+    copies = np.sort(pos.numpy())[:r]
+    for j, b in enumerate(rows):
+        if b % 2 == 0:
+            assert out["idx"][b].cpu().numpy().tolist() == copies.tolist()
+
+
 @pytest.mark.parametrize("N,d,B,r", [
     (200000, 128, 2048, 64),   # 8 query groups over 19 key ranges, two passes
     (70017, 64, 4000, 33),     # 16 groups (the last one partial), one pass
@@ -488,26 +567,35 @@ def _chunks(K, rows=65536):
         yield lo, synth.to_numpy_raw(K[lo:min(K.shape[0], lo + rows)])
 
 
-def test_large_batch_full_size_sampled_rows(nest):
-    """bf16 d=4096, N=4,194,304, B=512, r=256 (the benchmarked large-batch launch):
-    the oracle checks query rows 0 and 511 over all keys."""
-    w = synth.WORKLOADS["large_batch"]
-    x = synth.make_inputs(w, device="cuda")
-    ds = nest.Datastore(x.K, x.V, w.vocab)
-    out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam)
-    torch.cuda.synchronize()
-    assert ds.device_status() == 0
+def _oracle_rows_parallel(K, q_np, r, workers=16):
+    """The oracle's top-r of each row of q_np over all keys of the device tensor K:
+    distances chunk by chunk (the oracle's sqdist, OpenMP inside), then each
+    row's top-r (the oracle's topr) in a thread pool; the C calls release the
+    interpreter lock, so the per-row sorts run side by side."""
+    from concurrent.futures import ThreadPoolExecutor
+    B = q_np.shape[0]
+    D = np.empty((B, K.shape[0]), dtype=np.float64)
+    for lo, piece in _chunks(K):
+        D[:, lo:lo + piece.shape[0]] = oracle.sqdist(piece, q_np)
+    allidx = np.arange(K.shape[0], dtype=np.int64)
+    s = np.empty((B, r), dtype=np.float64)
+    idx = np.empty((B, r), dtype=np.int64)
+
+    def one(b):
+        Db, Ib, _ = oracle.topr(D[b], allidx, r)
+        s[b], idx[b] = -Db, Ib
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        list(ex.map(one, range(B)))
+    return s, idx
+
+
+def _check_rows_against(out, K, V, q_rows_np, rows, p_lm, w, s_or, i_or, label):
+    """Rows ``rows`` of a step's output against the oracle's (s_or, i_or) for
+    the same query vectors (row j of s_or belongs to output row rows[j])."""
     s_all, i_all = out["s"].cpu().numpy(), out["idx"].cpu().numpy()
-    qidx = [0, 511]
-    _check_rows_full_size_simple(out, x.K, x.V, x.q, qidx, x.p_lm, w, s_all, i_all)
-    ds.close()
-
-
-def _check_rows_full_size_simple(out, K, V, q, qidx, p_lm, w, s_all, i_all):
-    q_np = synth.to_numpy_raw(q[qidx])
-    s_or, i_or = oracle.knn_search_chunked(_chunks(K), q_np, w.r)
     V_np = V.cpu().numpy()
-    for j, b in enumerate(qidx):
+    p_m = out["p_m"].cpu().numpy()
+    for j, b in enumerate(rows):
         i_g = i_all[b]
         # exact distances of the union of both lists, from the rows themselves
         union = np.unique(np.concatenate([i_g, i_or[j]]))
@@ -515,33 +603,69 @@ def _check_rows_full_size_simple(out, K, V, q, qidx, p_lm, w, s_all, i_all):
         where = {int(k): n for n, k in enumerate(union)}
         g_loc = np.array([where[int(k)] for k in i_g])[None]
         o_loc = np.array([where[int(k)] for k in i_or[j]])[None]
-        rows = check_search(s_all[b:b + 1], g_loc, s_or[j:j + 1], o_loc, K_rows, q_np[j:j + 1],
-                            w.dtype, np.array([K.shape[0]]))
-        check_mix(out["p_m"][b:b + 1].cpu().numpy(), s_all[b:b + 1], i_all[b:b + 1], V_np,
-                  p_lm[b:b + 1].cpu().numpy(), w.mu, w.lam, w.vocab)
-        if rows:
+        matched = check_search(s_all[b:b + 1], g_loc, s_or[j:j + 1], o_loc, K_rows,
+                               q_rows_np[j:j + 1], w.dtype, np.array([K.shape[0]]), label=label)
+        p_lm_b = p_lm[b:b + 1].cpu().numpy()
+        check_mix(p_m[b:b + 1], s_all[b:b + 1], i_all[b:b + 1], V_np, p_lm_b, w.mu, w.lam,
+                  w.vocab)
+        if matched:
             P, n = oracle.pknn(s_or[j:j + 1], i_or[j:j + 1], V_np, w.mu, w.vocab)
-            ref = oracle.mix(p_lm[b:b + 1].cpu().numpy(), P, w.lam, n)
-            check_mix_end_to_end(out["p_m"][b:b + 1].cpu().numpy(), ref, [0])
+            ref = oracle.mix(p_lm_b, P, w.lam, n)
+            check_mix_end_to_end(p_m[b:b + 1], ref, [0])
+
+
+def _spread_rows(B, n, first=()):
+    """n distinct rows of a batch of B: the given first rows, then evenly spread."""
+    rows = list(first)
+    for v in np.linspace(0, B - 1, n).round().astype(int).tolist():
+        if len(rows) >= n:
+            break
+        if v not in rows:
+            rows.append(v)
+    k = 0
+    while len(rows) < n:
+        if k not in rows:
+            rows.append(k)
+        k += 1
+    return sorted(rows)
+
+
+def test_large_batch_full_size_sampled_rows(nest):
+    """bf16 d=4096, N=4,194,304, B=512, r=256 (the benchmarked large-batch launch):
+    the oracle checks 32 query rows spread over both query groups, over all keys."""
+    w = synth.WORKLOADS["large_batch"]
+    x = synth.make_inputs(w, device="cuda")
+    ds = nest.Datastore(x.K, x.V, w.vocab)
+    out = ds.step(x.q, w.r, x.p_lm, w.mu, w.lam)
+    torch.cuda.synchronize()
+    assert ds.device_status() == 0
+    rows = _spread_rows(512, 32, first=(0, 255, 256, 511))
+    q_np = synth.to_numpy_raw(x.q[rows])
+    s_or, i_or = _oracle_rows_parallel(x.K, q_np, w.r)
+    _check_rows_against(out, x.K, x.V, q_np, rows, x.p_lm, w, s_or, i_or,
+                        "config 4: large batch, 4M keys, B=512, r=256")
+    ds.close()
 
 
 def test_hidden8192_full_size_B_sweep(nest):
     """bf16 d=8192, N=8,388,608 clustered keys (128 GiB), r=1024, B in {1, 8, 64, 256}:
-    four kernel paths on one datastore.  Query 0 must get the same neighbours on
-    every path; the oracle checks queries 0 and 255 over all keys."""
+    four kernel paths on one datastore, each checked against the oracle on the
+    rows it shares with a fixed set of 32 rows (0-7, eight more below 64 and
+    sixteen spread to 255); the oracle scans all keys once for those rows."""
     w = synth.WORKLOADS["hidden8192"]
     x = synth.make_inputs(w, device="cuda", B=256)
     ds = nest.Datastore(x.K, x.V, w.vocab)
-    first = None
+    rows = sorted(set(range(8)) | {9, 17, 25, 33, 41, 49, 57, 63}
+                  | set(np.linspace(64, 255, 16).round().astype(int).tolist()))
+    assert len(rows) == 32
+    q_np = synth.to_numpy_raw(x.q[rows])
+    s_or, i_or = _oracle_rows_parallel(x.K, q_np, w.r)
     for B in (1, 8, 64, 256):
         out = ds.step(x.q[:B].contiguous(), w.r, x.p_lm[:B].contiguous(), w.mu, w.lam)
         torch.cuda.synchronize()
         assert ds.device_status() == 0, f"B={B}"
-        i0 = out["idx"][0].cpu().numpy()
-        if first is None:
-            first = i0
-        else:
-            assert set(first.tolist()) == set(i0.tolist()), f"B={B}: query 0 differs from B=1"
-    s_all, i_all = out["s"].cpu().numpy(), out["idx"].cpu().numpy()
-    _check_rows_full_size_simple(out, x.K, x.V, x.q, [0, 255], x.p_lm, w, s_all, i_all)
+        sel = [j for j, b in enumerate(rows) if b < B]
+        _check_rows_against(out, x.K, x.V, q_np[sel], [rows[j] for j in sel], x.p_lm, w,
+                            s_or[sel], i_or[sel],
+                            f"config 5: 8M keys, d=8192, r=1024, B={B}")
     ds.close()

@@ -45,13 +45,16 @@ def test_decode_plan(nest):
 
 def test_large_batch_plan(nest):
     """B=512, 4M keys, r=256: two groups of 256 queries, every key range once
-    per group in one wave (2 x 76 CTAs), thresholds from every 64th key
-    (65,536 = max(65,536, 256 r) sampled keys)."""
+    per group in one wave (2 x 76 CTAs), thresholds from every 60th key
+    (about max(65,536, 256 r') sampled keys, r' = 256 + 16 screened
+    candidates kept for the exact re-ranking)."""
+    rp = 256 + 16
     p = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM)
     assert p["kernel"] == "tc_wide2_kernel"
     assert (p["queries_per_group"], p["groups"], p["parts"]) == (256, 2, SMS // 2)
-    assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // 65536
-    assert p["list_capacity"] >= 8 * ((1 << 22) * 256 // 65536)  # 8x the expected survivors
+    assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // (256 * rp)
+    sample = (1 << 22) // p["sample_stride"]
+    assert p["list_capacity"] >= 8 * ((1 << 22) * rp // sample)  # 8x the expected survivors
     q = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
                           cta_pairs=True)
     assert q["kernel"] == "tc_wide_pair_kernel"
