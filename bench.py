@@ -1,14 +1,20 @@
 """Benchmark of the kNN-LM step (search + top-r + Eq. 2 + Eq. 3) on GB300.
 
-Default workload (``decode``): bf16 keys d=4096, N=1,048,576 from a 256-centre
-Gaussian mixture, values Zipf(1.1) over 32000 tokens, B=4 queries, r=1024,
-mu=1/64, lambda=0.8.  A step is one ``nest_knn_step`` over one batch.
+Default (headline) workload: the 70B-scale hidden size, bf16 keys d=8192,
+N=8,388,608 (128 GiB) from a 256-centre Gaussian mixture, values Zipf(1.1)
+over 32000 tokens, B=256 queries, r=1024, mu=1/sqrt(8192), lambda=0.8 -- the
+largest workload that fits one GPU, and the batch at which the HBM and the
+tensor-core rooflines meet.  A step is one ``nest_knn_step`` over one batch.
 
-Prints ONE JSON line (rank 0): queries/s over all ranks, the scan kernel's
-HBM roofline fraction (CUDA events around that kernel, inside the timed
+Prints ONE JSON line (rank 0): queries/s over all ranks, the dominant
+kernel's roofline fraction (CUDA events around that kernel, inside the timed
 region), the oracle timed on the host cores on a bounded sample, an
 end-to-end number through the public API with host buffers, and the SM
-clocks sampled during the timed region.
+clocks sampled during the timed region.  Its ``suite`` entry holds the other
+workloads measured in the same run, each with its own roofline and clocks:
+the same datastore at B = 1, 8 and 64, the decode batch (d=4096, 1M keys,
+B=4), the second-stage ragged search (32 x 10,240 keys) and the large batch
+(4M keys, B=512).
 
 ``--impl reference`` times the fp64 CPU oracle instead (the only reference
 implementation this method has here), on a bounded sample of the same
@@ -45,7 +51,8 @@ def parse():
     p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", default="decode", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--workload", default=None, choices=sorted(synth.WORKLOADS),
+                   help="one workload instead of the default headline + suite")
     p.add_argument("--B", type=int, default=None, help="override the query batch")
     p.add_argument("--N", type=int, default=None,
                    help="override the datastore size (small cases for profiling)")
@@ -63,7 +70,15 @@ def parse():
     p.add_argument("--sweep", default=None,
                    help="comma-separated query batch sizes measured on one datastore, one JSON "
                         "line each (e.g. 1,8,64,256 for the d=8192 workload)")
+    p.add_argument("--no-suite", action="store_true",
+                   help="headline workload only (no other workloads in the line)")
     return p.parse_args()
+
+
+# The headline workload and batch, and the other workloads measured with it.
+HEADLINE = ("hidden8192", 256)
+SUITE_SAME_DATASTORE = (64, 8, 1)  # further batches on the headline's datastore
+SUITE_OTHERS = (("decode", None), ("ragged", None), ("large_batch", None))
 
 
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
@@ -222,14 +237,17 @@ class OracleSampler:
                                  w.vocab, nthreads=self.threads)
         return time.perf_counter() - t0
 
-    def fit(self, budget_s: float) -> int:
-        """Largest key count (from a short calibration) whose sample fits the budget."""
+    def fit(self, budget_s: float, max_bytes: int = 4 << 30) -> int:
+        """Largest key count (from a short calibration) whose sample fits the
+        budget, at most ``max_bytes`` of keys copied to the host."""
         if self.ragged:
             return self.n
-        probe = min(self.n, 16384)
+        row = self.x.K.shape[1] * self.x.K.element_size()
+        cap = max(1024, max_bytes // row)
+        probe = min(self.n, 16384, cap)
         t = self.run(probe)
         n = int(probe * budget_s / max(t, 1e-6))
-        return max(min(self.n, n), min(self.n, 1024))
+        return max(min(self.n, n, cap), min(self.n, 1024))
 
     def queries_per_s(self, n: int, seconds: float) -> float:
         if self.ragged:
@@ -269,8 +287,23 @@ def cpu_model() -> str:
     return platform.machine()
 
 
+def oracle_queries_for(w, x, nq: int, budget_s: float) -> int:
+    """Queries of the oracle sample: more of them when the key sample is
+    capped by its size on the host, so that the sample still takes about
+    budget_s of CPU time (d=8192: 4 GiB are 262,144 keys)."""
+    if w.ragged:
+        return nq
+    row = x.K.shape[1] * x.K.element_size()
+    keys = min(x.K.shape[0], (4 << 30) // row)
+    # the oracle evaluates about 1.4e10 / d (query, key) distances per second on 16 cores
+    per_s = 1.4e10 / w.d * max(1, os.cpu_count() or 1) / 16
+    want = int(budget_s * per_s / keys)
+    return max(nq, min(x.q.shape[0], want))
+
+
 def cpu_baseline(w, x, nq: int, budget_s: float = 15.0):
     """The oracle on the host cores: one bounded sample of ~budget_s seconds."""
+    nq = oracle_queries_for(w, x, nq, budget_s)
     smp = OracleSampler(w, x, nq)
     n = smp.fit(budget_s)
     sec = smp.run(n)
@@ -279,15 +312,15 @@ def cpu_baseline(w, x, nq: int, budget_s: float = 15.0):
             "keys_per_s": smp.keys_per_s(n, sec), "cpu": cpu_model()}
 
 
-def run_reference(args, w, world, rank):
+def run_reference(args, w, B, world, rank):
     """``--impl reference``: the oracle on the host cores, each step a bounded sample."""
     if rank != 0:
         return
     dev = "cuda" if torch.cuda.is_available() else "cpu"
-    x = synth.make_inputs(w, device=dev, B=args.B, N=args.N)
-    nq = min(args.oracle_queries, x.q.shape[0])
+    x = synth.make_inputs(w, device=dev, B=B, N=args.N)
     total_steps = args.steps + args.warmup
     per_step = max(0.05, min(10.0, 150.0 / max(1, total_steps)))
+    nq = oracle_queries_for(w, x, min(args.oracle_queries, x.q.shape[0]), per_step)
     smp = OracleSampler(w, x, nq)
     n = smp.fit(per_step)
     times = []
@@ -313,33 +346,34 @@ def run_reference(args, w, world, rank):
     print(json.dumps(line), flush=True)
 
 
-# DRAM bytes (read + write) per launch of the dominant kernel, from one ncu
-# capture (dram__bytes_read.sum + dram__bytes_write.sum) of tc_scan_kernel on
-# a 65,536-key case, scaled to the default 1,048,576 keys (reads x16, per-CTA
-# writes unscaled).  Only valid for that kernel version on the default decode
-# workload.
-DECODE_TC_SCAN_TRAFFIC = 537.278464e6 * 16 + 3.055104e6
-
-# Same for the large-batch main pass (tc_wide2_kernel): a 262,144-key capture
-# scaled by 16 to the default 4,194,304 keys (key reads and, with the sample
-# size fixed at 65,536 keys, survivor writes both grow with N).  Only valid
-# for that kernel version on the default large batch.
-LARGE_BATCH_TC_WIDE2_TRAFFIC = (2.323294e9 + 28.291072e6) * 16
+# DRAM bytes (read + write) per launch of the dominant kernel, from ncu
+# captures (dram__bytes_read.sum + dram__bytes_write.sum) of that kernel on a
+# smaller case of the same workload, scaled to the full launch by the keys it
+# streams; only valid for the kernel versions captured.  None: not captured
+# for the current kernel.
+TRAFFIC = {}
 
 
-def dram_traffic(w, args, kernel):
-    if args.N is not None or args.B is not None:
+def dram_traffic(w, args, kernel, B):
+    if args.N is not None:
         return None
-    if w.name == "decode" and kernel == "tc_scan_kernel":
-        return DECODE_TC_SCAN_TRAFFIC
-    if w.name == "large_batch" and kernel == "tc_wide2_kernel":
-        return LARGE_BATCH_TC_WIDE2_TRAFFIC
-    return None
+    return TRAFFIC.get((w.name, kernel, B))
+
+
+DESCRIPTIONS = {
+    "tiny": "tiny exact kNN-LM step (fp32, d=64, 4,096 keys)",
+    "decode": "decode-batch full-datastore search (7B hidden size d=4096, 1,048,576 keys)",
+    "ragged": "two-stage ragged search (NEST second stage, 40 passages x 256 keys per query)",
+    "large_batch": "large-batch prefill-style search (d=4096, 4,194,304 keys)",
+    "nest_span": "span verification batch over one query's K' (40 passages x 256 keys)",
+    "hidden8192": "70B-scale hidden size (d=8192, 8,388,608 keys, 128 GiB)",
+}
 
 
 def config_of(w, x, pipeline="knnlm"):
     B = x.q.shape[0]
-    return {"workload": w.name, "pipeline": pipeline, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
+    return {"workload": w.name, "description": DESCRIPTIONS.get(w.name, w.name),
+            "pipeline": pipeline, "N": int(x.K.shape[0]), "d": w.d, "B": int(B), "r": w.r,
             "vocab": w.vocab, "key_dtype": w.dtype, "accumulate": "f32",
             "mu": w.mu, "lambda": w.lam,
             "ragged": bool(w.ragged),
@@ -348,10 +382,19 @@ def config_of(w, x, pipeline="knnlm"):
 
 def main():
     args = parse()
-    w = synth.WORKLOADS[args.workload]
     world, rank, local = dist_setup()
+    if args.workload is None:
+        name, B_head = HEADLINE
+        suite = (not args.no_suite and args.sweep is None and args.pipeline == "knnlm"
+                 and args.N is None and args.B is None)
+    else:
+        name, B_head = args.workload, None
+        suite = False
+    if args.B is not None:
+        B_head = args.B
+    w = synth.WORKLOADS[name]
     if args.impl == "reference":
-        run_reference(args, w, world, rank)
+        run_reference(args, w, B_head, world, rank)
         return
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA GPU for the CUDA path")
@@ -361,17 +404,39 @@ def main():
     nest_build.build()
 
     dev = torch.device("cuda", local)
-    sweep = [int(v) for v in args.sweep.split(",")] if args.sweep else [args.B]
+    sweep = [int(v) for v in args.sweep.split(",")] if args.sweep else [B_head]
     B_gen = max(b for b in sweep if b is not None) if any(b is not None for b in sweep) else None
     x = synth.make_inputs(w, device=dev, B=B_gen, N=args.N, seed=w.seed + rank)
     ds = nest.Datastore(x.K, x.V, w.vocab)
     if args.cta_pairs:
         ds.use_cta_pairs(True)
+    lines = []
     for B in sweep:
-        line = measure(args, w, x, ds, B if B is not None else x.q.shape[0], world, rank, local)
+        lines.append(measure(args, w, x, ds, B if B is not None else x.q.shape[0], world, rank,
+                             local))
+        if rank == 0 and not suite:
+            print(json.dumps(lines[-1]), flush=True)
+    if suite:
+        extras = {}
+        for B in SUITE_SAME_DATASTORE:
+            extras[f"{w.name}_B{B}"] = measure(args, w, x, ds, B, world, rank, local, light=True)
+        ds.close()
+        del ds, x
+        torch.cuda.empty_cache()
+        for oname, oB in SUITE_OTHERS:
+            ow = synth.WORKLOADS[oname]
+            ox = synth.make_inputs(ow, device=dev, B=oB, seed=ow.seed + rank)
+            ods = nest.Datastore(ox.K, ox.V, ow.vocab)
+            extras[oname] = measure(args, ow, ox, ods, ox.q.shape[0], world, rank, local,
+                                    light=True)
+            ods.close()
+            del ods, ox
+            torch.cuda.empty_cache()
         if rank == 0:
-            print(json.dumps(line), flush=True)
-    ds.close()
+            lines[0]["suite"] = extras
+            print(json.dumps(lines[0]), flush=True)
+    else:
+        ds.close()
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
@@ -446,8 +511,11 @@ def graph_replay(step, stream, args, world, B):
     return {"ms_per_step": ms, "value": world * B / (ms / 1e3), "steps": n}
 
 
-def measure(args, w, x_all, ds, B, world, rank, local):
-    """Time one batch size on an existing datastore; returns the JSON line (rank 0)."""
+def measure(args, w, x_all, ds, B, world, rank, local, light=False):
+    """Time one batch size on an existing datastore; returns the JSON line (rank 0).
+
+    ``light``: a suite entry (value, roofline, clocks, e2e, launches), without
+    the CPU baseline, the CUDA-graph replays and the search-only timing."""
     x = synth.Inputs(K=x_all.K, V=x_all.V, q=x_all.q[:B].contiguous(),
                      p_lm=x_all.p_lm[:B].contiguous(),
                      seg_off=x_all.seg_off[:B + 1].contiguous() if x_all.seg_off is not None else None)
@@ -485,6 +553,7 @@ def measure(args, w, x_all, ds, B, world, rank, local):
         raise SystemExit("device status error during the timed steps")
     ms = max_over_ranks(ms_local, world)
     value = aggregate(world, B, args.steps, ms)
+    step_ms = ms / args.steps
 
     # ---- roofline of the dominant kernel (the key scan)
     esize = 2 if w.dtype == "bf16" else 4
@@ -501,48 +570,52 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     t_hbm = alg_bytes / (hbm_peak * 1e9)
     t_tc = alg_flops / (tc_peak * 1e12)
     kernel = ds.search_path(B, w.r, ragged=x.seg_off is not None)
+    hbm_frac = alg_bytes / (scan_avg_ms / 1e3) / 1e9 / hbm_peak
+    tensor_frac = alg_flops / (scan_avg_ms / 1e3) / 1e12 / tc_peak
+    common = {"traffic": dram_traffic(w, args, kernel, B), "kernel": kernel,
+              "alg_flops_per_launch": alg_flops, "alg_bytes_per_launch": alg_bytes,
+              "hbm_frac": hbm_frac, "tensor_frac": tensor_frac,
+              "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
+    if clk and clk.get("sm_mhz"):
+        # the power cap moves the SM clock in tensor-bound runs: time x clock
+        common["launch_ms_x_sm_ghz"] = scan_avg_ms * clk["sm_mhz"] / 1e3
     if t_tc > t_hbm:
         achieved = alg_flops / (scan_avg_ms / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s",
-                    "frac": achieved / tc_peak, "traffic": dram_traffic(w, args, kernel),
-                    "kernel": kernel, "peak_kind": peak_kind + " (bf16 dense, sustained)",
-                    "alg_flops_per_launch": alg_flops, "alg_bytes_per_launch": alg_bytes,
-                    "hbm_frac": alg_bytes / (scan_avg_ms / 1e3) / 1e9 / hbm_peak,
-                    "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
+                    "frac": achieved / tc_peak,
+                    "peak_kind": peak_kind + " (bf16 dense, sustained)", **common}
     else:
         achieved = alg_bytes / (scan_avg_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                    "frac": achieved / hbm_peak, "traffic": dram_traffic(w, args, kernel),
-                    "kernel": kernel, "peak_kind": peak_kind,
-                    "alg_bytes_per_launch": alg_bytes, "alg_flops_per_launch": alg_flops,
-                    "tensor_frac": alg_flops / (scan_avg_ms / 1e3) / 1e12 / tc_peak,
-                    "launch_ms": scan_avg_ms, "share_of_step": scan_ms / ms_local}
+                    "frac": achieved / hbm_peak, "peak_kind": peak_kind, **common}
 
-    # ---- the same step captured once in a CUDA graph and replayed
-    graph = graph_replay(step, stream, args, world, B)
-    if ds.device_status() != 0:
-        raise SystemExit("device status error during the graph replays")
+    graph = search = None
+    if not light:
+        # ---- the same step captured once in a CUDA graph and replayed
+        graph = graph_replay(step, stream, args, world, B)
+        if ds.device_status() != 0:
+            raise SystemExit("device status error during the graph replays")
 
-    # ---- the search alone (scan and merge or selection, no mix), same batch
-    s_buf = torch.empty(B, w.r, dtype=torch.float32, device=x.q.device)
-    i_buf = torch.empty(B, w.r, dtype=torch.int64, device=x.q.device)
-    n_search = max(1, min(args.steps, 200))
-    for _ in range(3):
-        ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
-    barrier(world)
-    torch.cuda.synchronize()
-    u0 = torch.cuda.Event(enable_timing=True)
-    u1 = torch.cuda.Event(enable_timing=True)
-    u0.record(stream)
-    for _ in range(n_search):
-        ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
-    u1.record(stream)
-    torch.cuda.synchronize()
-    search_ms = max_over_ranks(u0.elapsed_time(u1), world) / n_search
-    if ds.device_status() != 0:
-        raise SystemExit("device status error during the search-only steps")
-    search = {"call": "nest_knn_search", "ms": search_ms,
-              "queries_per_s": world * B / (search_ms / 1e3), "steps": n_search}
+        # ---- the search alone (scan, merge or selection, re-ranking; no mix), same batch
+        s_buf = torch.empty(B, w.r, dtype=torch.float32, device=x.q.device)
+        i_buf = torch.empty(B, w.r, dtype=torch.int64, device=x.q.device)
+        n_search = max(1, min(args.steps, 200))
+        for _ in range(3):
+            ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
+        barrier(world)
+        torch.cuda.synchronize()
+        u0 = torch.cuda.Event(enable_timing=True)
+        u1 = torch.cuda.Event(enable_timing=True)
+        u0.record(stream)
+        for _ in range(n_search):
+            ds.search(x.q, w.r, seg_off=x.seg_off, s_out=s_buf, idx_out=i_buf)
+        u1.record(stream)
+        torch.cuda.synchronize()
+        search_ms = max_over_ranks(u0.elapsed_time(u1), world) / n_search
+        if ds.device_status() != 0:
+            raise SystemExit("device status error during the search-only steps")
+        search = {"call": "nest_knn_search", "ms": search_ms,
+                  "queries_per_s": world * B / (search_ms / 1e3), "steps": n_search}
 
     # ---- end to end through the public API with pinned host buffers
     q_h = x.q.cpu().pin_memory()
@@ -569,16 +642,27 @@ def measure(args, w, x_all, ds, B, world, rank, local):
             res_h.copy_(step(), non_blocking=True)
             stream.synchronize()
         d2h = res_h.numel() * res_h.element_size()
+    # about three seconds of end-to-end steps at most (and at least five)
+    n_e2e = max(5, min(args.e2e_steps, int(3000.0 / max(step_ms, 1e-3))))
     for _ in range(3):
         e2e_step()
     barrier(world)
     te = time.perf_counter()
-    for _ in range(args.e2e_steps):
+    for _ in range(n_e2e):
         e2e_step()
     e2e_s = max_over_ranks(time.perf_counter() - te, world)
-    e2e = {"value": world * B * args.e2e_steps / e2e_s,
+    e2e = {"value": world * B * n_e2e / e2e_s,
            "unit": "positions/s" if args.pipeline == "verify" else "queries/s",
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e}
+
+    unit = "positions/s" if args.pipeline == "verify" else "queries/s"
+    if light:
+        if rank != 0:
+            return None
+        return {"value": value, "unit": unit, "ms_per_step": step_ms,
+                "config": config_of(w, x, args.pipeline),
+                "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
+                "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clk}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -588,9 +672,9 @@ def measure(args, w, x_all, ds, B, world, rank, local):
     line = None
     if rank == 0:
         line = {
-            "metric": metric, "value": value,
-            "unit": "positions/s" if args.pipeline == "verify" else "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "metric": metric, "value": value, "unit": unit, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
             "data": "synthetic", "config": config_of(w, x, args.pipeline),
             "keys_scanned_per_s": world * keys_scanned * args.steps / (ms / 1e3),
