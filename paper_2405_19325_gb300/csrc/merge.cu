@@ -44,6 +44,8 @@ __global__ void __launch_bounds__(kMergeThreads, 1) merge_kernel(const MergeArgs
     extern __shared__ __align__(16) unsigned char smem[];
     uint64_t* buf = reinterpret_cast<uint64_t*>(smem);
     MergeShared& sh = *reinterpret_cast<MergeShared*>(smem + buf_words(a.per_cta, a.r) * 8);
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int b = blockIdx.y, grp = blockIdx.x;
     const int l0 = grp * a.per_cta;
@@ -145,8 +147,7 @@ cudaError_t launch_merge(const MergeArgs& a, cudaStream_t stream)
     const dim3 grid(groups, a.B);
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(merge_kernel), (int)smem);
     if (e != cudaSuccess) return e;
-    merge_kernel<<<grid, kMergeThreads, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(merge_kernel, grid, dim3(kMergeThreads), smem, stream, a);
 }
 
 }  // namespace nest

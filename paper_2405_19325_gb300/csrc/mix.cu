@@ -62,6 +62,8 @@ __global__ void __launch_bounds__(kMixThreads) mix_kernel(const MixArgs a)
     __shared__ float bc[4];
     __shared__ int bci;
 
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int b = blockIdx.y, slice = blockIdx.x;
     // Slice boundaries fall on multiples of 4 when the vocabulary allows it.
@@ -210,8 +212,7 @@ cudaError_t launch_mix(const MixArgs& a, cudaStream_t stream)
         raise_smem_limit(reinterpret_cast<const void*>(mix_kernel), (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid(a.slices, a.B);
-    mix_kernel<<<grid, kMixThreads, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(mix_kernel, grid, dim3(kMixThreads), smem, stream, a);
 }
 
 int mix_min_slices(int vocab) { return (vocab + kMixMaxSliceTokens - 1) / kMixMaxSliceTokens; }

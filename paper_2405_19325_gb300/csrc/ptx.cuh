@@ -14,6 +14,22 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p)
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization (launch_pdl) may be scheduled while the kernel before it in
+// the stream is still running; grid_dependency_wait() blocks until that
+// kernel has completed and its memory writes are visible (for an ordinary
+// launch it returns at once).  Every kernel of the library calls it before
+// it reads or writes global memory.  grid_dependents_launch() lets the next
+// kernel be scheduled from now on (it still waits for this one to finish).
+__device__ __forceinline__ void grid_dependency_wait()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependents_launch()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t global_timer_ns()
 {
     uint64_t t;

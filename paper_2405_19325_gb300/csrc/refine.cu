@@ -14,10 +14,11 @@
 // then keeps the r nearest by those distances (ties: smaller key index),
 // sorts them and writes s = -distance and the key index.
 //
-// Grid (chunks of 32 candidates, B queries), 1024 threads: warp w of chunk c
-// recomputes candidate 32 c + w.  A CTA rewrites its candidates' words in
-// place, and the last CTA of a query to finish (an atomic counter, no wait)
-// selects, sorts and writes the row.
+// Grid (chunks of 16 candidates, B queries), 512 threads: warp w of chunk c
+// recomputes candidate 16 c + w, eight 16-byte loads in flight per lane.  A
+// CTA rewrites its candidates' words in place, and the last CTA of a query
+// to finish (an atomic counter, no wait) sorts the r' words (bitonic, in
+// shared memory) and writes the first r.
 //
 // It also checks the margin.  A key left out of the r' candidates had a
 // screened distance of at least A, the largest screened distance kept.  The
@@ -42,8 +43,9 @@
 namespace nest {
 namespace {
 
-constexpr int kRefineThreads = 1024;
+constexpr int kRefineThreads = 512;
 constexpr int kRefineRows = kRefineThreads / 32;  // candidates per CTA
+constexpr int kRefineLoads = 8;                   // 16-byte loads in flight per lane
 // Distance bits no real distance has (a NaN pattern above +inf's bits).
 constexpr uint64_t kPadHigh = 0xFFFFFFFFull << 32;
 
@@ -62,9 +64,6 @@ struct RefineShared {
     uint32_t emax, emin;      // largest / smallest screened - exact distance (ordered bits)
     unsigned long long apair; // largest (screened bits << 32 | exact bits) of this CTA
     int last;
-    int cnt;
-    uint64_t thr;
-    SelectSmem<kRefineThreads, 1> sel;
 };
 
 __host__ __device__ inline int pow2_at_least(int x)
@@ -99,12 +98,14 @@ __device__ __forceinline__ void chunk_sqdiff(const uint4& k, const uint4& q, flo
 }
 
 template <int DT>
-__global__ void __launch_bounds__(kRefineThreads, 1) refine_kernel(const RefineArgs a)
+__global__ void __launch_bounds__(kRefineThreads) refine_kernel(const RefineArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     uint4* qs = reinterpret_cast<uint4*>(smem);  // the query row
     uint64_t* buf = reinterpret_cast<uint64_t*>(smem + a.row_bytes);
     __shared__ RefineShared sh;
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int b = blockIdx.y;
     const int chunks = a.row_bytes / 16;
@@ -131,12 +132,12 @@ __global__ void __launch_bounds__(kRefineThreads, 1) refine_kernel(const RefineA
                 static_cast<const unsigned char*>(a.K) + (size_t)key * a.row_bytes);
             float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
             int c = lane;
-            for (; c + 3 * 32 < chunks; c += 4 * 32) {
-                uint4 kv[4];
+            for (; c + (kRefineLoads - 1) * 32 < chunks; c += kRefineLoads * 32) {
+                uint4 kv[kRefineLoads];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) kv[u] = ld_global_nc_v4(krow + c + 32 * u);
+                for (int u = 0; u < kRefineLoads; ++u) kv[u] = ld_global_nc_v4(krow + c + 32 * u);
 #pragma unroll
-                for (int u = 0; u < 4; ++u) chunk_sqdiff<DT>(kv[u], qs[c + 32 * u], acc);
+                for (int u = 0; u < kRefineLoads; ++u) chunk_sqdiff<DT>(kv[u], qs[c + 32 * u], acc);
             }
             for (; c < chunks; c += 32) chunk_sqdiff<DT>(ld_global_nc_v4(krow + c), qs[c], acc);
             float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
@@ -167,30 +168,26 @@ __global__ void __launch_bounds__(kRefineThreads, 1) refine_kernel(const RefineA
     if (!sh.last) return;
     __threadfence();
 
-    // ---- last CTA of this query: r nearest by exact distance, sorted.  A
-    // padding word (none is expected among the n) becomes a distinct word
-    // above every real one, so the select sees distinct words.
-    for (int i = tid; i < n; i += kRefineThreads) {
-        const uint64_t w = __ldcg(list + i);
-        buf[i] = w != kNoCandidate ? w : (kPadHigh | (uint32_t)i);
+    // ---- last CTA of this query: all candidates sorted by exact distance
+    // (ties: smaller key index), the first r written.  A padding word (none
+    // is expected among the n) becomes a distinct word above every real one.
+    const int P2 = pow2_at_least(n > 0 ? n : 1);
+    for (int i = tid; i < P2; i += kRefineThreads) {
+        uint64_t w = kNoCandidate;
+        if (i < n) {
+            w = __ldcg(list + i);
+            if (w == kNoCandidate) w = kPadHigh | (uint32_t)i;
+        }
+        buf[i] = w;
     }
-    if (tid == 0) {
-        sh.cnt = n;
-        sh.thr = kNoCandidate;
-    }
-    __syncthreads();
-    select_smallest<kRefineThreads, 1>(buf, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
-                                       [] { __syncthreads(); });
-    const int m = sh.cnt;
-    const int P2 = pow2_at_least(m > 0 ? m : 1);
-    for (int i = m + tid; i < P2; i += kRefineThreads) buf[i] = kNoCandidate;
     __syncthreads();
     bitonic_sort<kRefineThreads>(buf, P2, tid, [] { __syncthreads(); });
+    const int m = n < a.r ? n : a.r;
     float* so = a.s_out + (int64_t)b * a.r;
     int64_t* io = a.idx_out + (int64_t)b * a.r;
     for (int i = tid; i < a.r; i += kRefineThreads) {
         const uint64_t e = i < m ? buf[i] : kNoCandidate;
-        if ((e >> 32) != 0xFFFFFFFFu) {
+        if ((e >> 32) < 0xFFFFFFFFu) {
             so[i] = -__uint_as_float((uint32_t)(e >> 32));
             io[i] = (int64_t)(uint32_t)e;
         } else {
@@ -224,23 +221,22 @@ int refine_margin(int r)
 
 size_t refine_smem_bytes(int rp, int r, int row_bytes)
 {
-    const int words = rp > pow2_at_least(r) ? rp : pow2_at_least(r);
-    return (size_t)row_bytes + (size_t)words * sizeof(uint64_t);
+    (void)r;
+    return (size_t)row_bytes + (size_t)pow2_at_least(rp) * sizeof(uint64_t);
 }
 
 cudaError_t launch_refine(int dtype, const RefineArgs& a, cudaStream_t stream)
 {
     const dim3 grid((a.rp + kRefineRows - 1) / kRefineRows, a.B);
     const size_t smem = refine_smem_bytes(a.rp, a.r, a.row_bytes);
-    const void* kern = dtype == NEST_BF16 ? reinterpret_cast<const void*>(refine_kernel<NEST_BF16>)
-                                          : reinterpret_cast<const void*>(refine_kernel<NEST_F32>);
-    cudaError_t e = raise_smem_limit(kern, smem);
+    if (dtype == NEST_BF16) {
+        cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(refine_kernel<NEST_BF16>), smem);
+        if (e != cudaSuccess) return e;
+        return launch_pdl(refine_kernel<NEST_BF16>, grid, dim3(kRefineThreads), smem, stream, a);
+    }
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(refine_kernel<NEST_F32>), smem);
     if (e != cudaSuccess) return e;
-    if (dtype == NEST_BF16)
-        refine_kernel<NEST_BF16><<<grid, kRefineThreads, smem, stream>>>(a);
-    else
-        refine_kernel<NEST_F32><<<grid, kRefineThreads, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(refine_kernel<NEST_F32>, grid, dim3(kRefineThreads), smem, stream, a);
 }
 
 }  // namespace nest

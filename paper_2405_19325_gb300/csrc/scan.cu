@@ -134,6 +134,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) scan_topr_kernel(const ScanAr
     static_assert(NV <= 32 && (NV & (NV - 1)) == 0, "NV must be a power of two <= 32");
 
     extern __shared__ __align__(128) unsigned char smem[];
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int item = blockIdx.x;
     const int group = item / a.parts, part = item - group * a.parts;
@@ -409,8 +411,7 @@ cudaError_t launch_impl(const ScanPlan& p, const ScanArgs& a, cudaStream_t strea
     auto kern = scan_topr_kernel<DT, NQ, CPT>;
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.groups * p.parts, kScanThreads, p.smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kScanThreads), p.smem, stream, a);
 }
 
 template <int DT, int NQ>

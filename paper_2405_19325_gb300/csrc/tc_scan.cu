@@ -82,6 +82,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* cand = reinterpret_cast<uint64_t*>(smem + (size_t)a.stages * kStageBytes);
     TcShared<NQ>& sh = *reinterpret_cast<TcShared<NQ>*>(cand + (size_t)NQ * a.cap);
 
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int item = blockIdx.x;
     const int group = item / a.parts, part = item - group * a.parts;
@@ -300,8 +302,8 @@ cudaError_t tc_launch_nq(const TcPlan& p, const CUtensorMap& tmK, const CUtensor
     cudaError_t e =
         raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kTcThreads), p.smem, stream, tmK, tmQ,
+                      a);
 }
 
 }  // namespace

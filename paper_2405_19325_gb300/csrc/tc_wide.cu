@@ -363,6 +363,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     unsigned char* stages = smem;
     WideShared<NM>& sh = *reinterpret_cast<WideShared<NM>*>(smem + (size_t)a.stages * kStage);
 
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     // CTAs of the same key range but different query groups are adjacent, so
     // they stream the same tiles at about the same time and share them in L2.
@@ -562,6 +564,8 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
     unsigned char* stages = smem;
     WideShared<NM>& sh = *reinterpret_cast<WideShared<NM>*>(smem + (size_t)a.stages * kStage);
 
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int part = blockIdx.x / a.groups, group = blockIdx.x - part * a.groups;
     const int q0 = group * NM;
@@ -918,6 +922,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
 __global__ void __launch_bounds__(256) wide_qnorm_kernel(const unsigned char* q, int32_t B,
                                                          int32_t d, float* qn)
 {
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int lane = threadIdx.x & 31;
     const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
     if (j >= B) return;
@@ -1001,6 +1007,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
 {
     extern __shared__ __align__(16) uint64_t stage[];  // a.stage_words words
     __shared__ GselShared sh;
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int q = blockIdx.x;
     uint64_t* list = a.cand + (int64_t)q * a.cap;
@@ -1230,15 +1238,15 @@ cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUte
     if (NM == 256 && p.mb == 2) {
         cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_wide2_kernel), (int)p.smem);
         if (e != cudaSuccess) return e;
-        tc_wide2_kernel<<<p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ, a);
-        return cudaGetLastError();
+        return launch_pdl(tc_wide2_kernel, dim3(p.groups * p.parts), dim3(kWide2Threads), p.smem,
+                          stream, tmK, tmQ, a);
     }
     auto kern = tc_wide_kernel<NM>;
     cudaError_t e =
         raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kTcThreads), p.smem, stream, tmK, tmQ,
+                      a);
 }
 
 }  // namespace
@@ -1302,8 +1310,8 @@ cudaError_t recover_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const C
     auto kern = tc_wide_kernel<NM, true>;
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kTcThreads), p.smem, stream, tmK, tmQ,
+                      a);
 }
 
 }  // namespace
@@ -1348,9 +1356,8 @@ cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUte
 
 cudaError_t launch_wide_qnorm(const void* q, int32_t B, int32_t d, float* qn, cudaStream_t stream)
 {
-    wide_qnorm_kernel<<<(B + 7) / 8, 256, 0, stream>>>(static_cast<const unsigned char*>(q), B, d,
-                                                       qn);
-    return cudaGetLastError();
+    return launch_pdl(wide_qnorm_kernel, dim3((B + 7) / 8), dim3(256), 0, stream,
+                      static_cast<const unsigned char*>(q), B, d, qn);
 }
 
 cudaError_t launch_gselect(const GselectArgs& in, cudaStream_t stream)
@@ -1362,8 +1369,7 @@ cudaError_t launch_gselect(const GselectArgs& in, cudaStream_t stream)
     const size_t smem = (size_t)a.stage_words * sizeof(uint64_t);
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(gselect_kernel), (int)smem);
     if (e != cudaSuccess) return e;
-    gselect_kernel<<<a.B, kSelThreads, smem, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(gselect_kernel, dim3(a.B), dim3(kSelThreads), smem, stream, a);
 }
 
 }  // namespace nest
