@@ -352,14 +352,10 @@ def run_reference(args, w, B, world, rank):
 # streams; only valid for the kernel versions captured.  None: not captured
 # for the current kernel.
 TRAFFIC = {
-    # tc_wide2_kernel main pass, d=8192, B=256: a 557,056-key capture, x 8,388,608 / 557,056
-    ("hidden8192", "tc_wide2_kernel", 256): (9151764480 + 22434816) * 8388608 / 557056,
     # tc_scan_kernel<4>, decode: a 65,536-key capture; reads x16, per-CTA list writes as they are
     ("decode", "tc_scan_kernel", 4): 537274880 * 16 + 2926080,
     # tc_scan_kernel<1>, ragged: captured at full size
     ("ragged", "tc_scan_kernel", 32): 2686010112 + 2874880,
-    # tc_wide2_kernel main pass, large batch: a 262,144-key capture, x16
-    ("large_batch", "tc_wide2_kernel", 512): (2319727104 + 27057664) * 16,
 }
 
 

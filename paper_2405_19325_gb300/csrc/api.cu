@@ -50,7 +50,7 @@ namespace {
 constexpr int64_t kMaxKeys = 4294967294LL;  // key indices travel as 32 bits
 // Recovery passes after an overflowed large-batch list (each at most one
 // more scan of the keys, only for the query groups concerned).
-constexpr int kRecoverRounds = 2;
+constexpr int kRecoverRounds = 3;
 constexpr int32_t kMaxB = 65535;
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -86,6 +86,7 @@ struct SearchPlan {
     bool wide;
     WidePlan wps, wpm, wpr;   // sample pass, main pass, recovery pass
     int64_t stride;           // sample = every stride-th key
+    int32_t thr_rank;         // main pass admits keys up to the sample's thr_rank-th distance
     int64_t sample_rows;
     bool single_pass;         // the sample is the whole datastore
     int64_t cap_s, cap_m;     // list capacities per query
@@ -189,16 +190,22 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
         WidePlan wp{};
         if (wide_plan_smem(nm, ds->smem_optin, ds->pairs, &wp)) {
             wp.groups = (B + nm - 1) / nm;
-            // Sample of about max(65,536, k r) keys, so that at most a
-            // fraction 1/k of the keys survives its r-th distance.  Groups of
-            // 256 queries run a tensor-bound main pass whose epilogue the
-            // survivors slow down (k = 256); smaller batches gain more from a
-            // cheaper sampling pass and selection (k = 64).
-            const int64_t k = nm == 256 ? 256 : 64;
-            const int64_t target = std::max<int64_t>(65536, k * r);
+            // A sample of every stride-th key, about max(65,536, 64 r) keys.
+            const int64_t target = std::max<int64_t>(65536, 64 * (int64_t)r);
             sp->stride = std::max<int64_t>(1, ds->N / target);
             sp->sample_rows = ds->N / sp->stride;
             sp->single_pass = sp->stride == 1;
+            // Admission threshold of the main pass: the sample's j-th
+            // smallest distance.  The sample holds on average r / stride of
+            // a query's r nearest keys; j = max(32, 4 r / stride) lets about
+            // max(32 stride, 4 r) keys of the datastore through, and the
+            // chance that the sample holds j of the r nearest (so that fewer
+            // than r keys pass) is negligible for any layout that systematic
+            // sampling does not alias.  It is checked all the same: a query
+            // left with fewer than r survivors is scanned again with the
+            // sample's r-th distance, which bounds the true r-th from above.
+            sp->thr_rank = (int32_t)std::min<int64_t>(
+                r, std::max<int64_t>(32, (4 * (int64_t)r + sp->stride - 1) / sp->stride));
             sp->wps = wp;
             // a CTA pair takes two SMs
             const int slots = wp.pair ? ds->num_sms / 2 : ds->num_sms;
@@ -206,19 +213,21 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
             sp->wpm = wp;
             sp->wpm.parts = choose_parts(wp.groups, ds->N, slots, false);
             sp->cap_s = sp->sample_rows;
-            const int64_t expect = (ds->N * (int64_t)r + sp->sample_rows - 1) / sp->sample_rows;
+            const int64_t expect =
+                (ds->N * (int64_t)sp->thr_rank + sp->sample_rows - 1) / sp->sample_rows;
             // Main-pass lists hold 8x the expected survivors plus what the
             // epilogue warps' reservations can leave unwritten.  About a
-            // fraction r / sample_rows of the keys pass the sample's r-th
+            // fraction j / sample_rows of the keys pass the sample's j-th
             // distance, so a warp that drains `rows` key rows admits about
-            // rows * r / sample_rows keys per query; it reserves twice that
+            // rows * j / sample_rows keys per query; it reserves twice that
             // plus 16 slots at a time (one atomic per block).  Each column
             // has 4 reserving warps per CTA (8 with two key tiles per stage).
             const int epi_warps = wp.mb == 2 ? 8 : 4;
             const int64_t unit = (int64_t)kTcTileKeys * wp.mb;
             const int64_t units = (ds->N + unit - 1) / unit;
             const int64_t rows = (units + sp->wpm.parts - 1) / sp->wpm.parts * 32;
-            const int64_t per_warp = (rows * r + sp->sample_rows - 1) / sp->sample_rows;
+            const int64_t per_warp =
+                (rows * sp->thr_rank + sp->sample_rows - 1) / sp->sample_rows;
             sp->resv = (int32_t)std::min<int64_t>(2 * per_warp + 16, 1024);
             const int64_t unwritten = (int64_t)sp->wpm.parts * epi_warps * sp->resv;
             sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect)) + unwritten;
@@ -525,8 +534,9 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     ga.idx_out = i_s;
     e = launch_gselect(ga, stream);
     if (e != cudaSuccess) return from_cuda(e);
-    // 2. every key, admitted at or below the sample's r-th screened distance
+    // 2. every key, admitted at or below the sample's thr_rank-th screened distance
     wa.s_sample = s_s;
+    wa.thr_rank = sp.thr_rank;
     wa.cand = scratch + sp.off_cand_m;
     wa.cnt = cnt + B;
     wa.cap = sp.cap_m;
@@ -538,10 +548,12 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     e = launch_tc_wide(sp.wpm, ds->keys_map, qmap, wa, stream);
     if (e != cudaSuccess) return from_cuda(e);
     if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
-    // 3. lists that overflowed (more survivors than their capacity: many
-    // keys tied at the sample's threshold, say) are scanned again with a
-    // tighter limit: the r-th smallest word each holds.  Both kernels of a
-    // round return at once when no list needs it.
+    // 3. Lists with fewer than r survivors (the threshold came out below
+    // the query's r-th distance) are scanned again up to the sample's r-th
+    // distance, a safe bound; lists that overflowed (more survivors than
+    // their capacity: many keys tied at the threshold, say) are scanned
+    // again with a tighter limit, the r-th smallest word each holds.  Both
+    // kernels of a round return at once when no list needs it.
     uint64_t* lim = scratch + sp.off_lim;
     CUtensorMap rmap;
     if (!encode_bf16_rows(&rmap, q, B, ds->d, sp.wpr.nm, false)) return NEST_ERR_CUDA;
@@ -555,6 +567,8 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
         gp.lim_out = lim;
         gp.group_flag = flags + (size_t)round * sp.wpm.groups;
         gp.group_size = sp.wpm.nm;
+        gp.s_sample = s_s;
+        gp.check_underflow = round == 0 ? 1 : 0;
         e = launch_gselect(gp, stream);
         if (e != cudaSuccess) return from_cuda(e);
         WideArgs wr = wa;

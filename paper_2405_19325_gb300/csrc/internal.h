@@ -160,8 +160,9 @@ struct WideArgs {
     const float* qn;  // B: ||q||^2 (launch_wide_qnorm)
     const uint32_t* key_mask;  // nullptr, or bit k set: key k is never a candidate
     int* status;
-    const float* s_sample;  // B x r sample neighbours (threshold = s[r-1]); null: admit all
+    const float* s_sample;  // B x r sample neighbours (threshold = s[thr_rank-1]); null: admit all
     int32_t r;
+    int32_t thr_rank;       // 1 <= thr_rank <= r
     uint64_t* cand;  // [B][cap] candidate words
     int32_t* cnt;    // [B] candidates appended (must start at 0)
     int64_t cap;
@@ -198,11 +199,16 @@ struct GselectArgs {
     unsigned long long* refine_apair;
     int* status;          // with words_out: NEST_ERR_OVERFLOW if a list is still over capacity
     // Recovery preparation (instead of any output): for an overflowed list,
-    // lim_out[q] = the r-th smallest word it holds, cnt[q] = 0 and
-    // group_flag[q / group_size] = 1; for a complete list lim_out[q] = kNoCandidate.
+    // lim_out[q] = the r-th smallest word it holds; for a list with fewer
+    // than r real words (when check_underflow), lim_out[q] = every word up to
+    // the sample's r-th distance s_sample[q * r + r - 1]; for either,
+    // cnt[q] = 0 and group_flag[q / group_size] = 1.  Otherwise
+    // lim_out[q] = kNoCandidate.
     uint64_t* lim_out;
     int32_t* group_flag;
     int32_t group_size;
+    const float* s_sample;
+    int32_t check_underflow;
     int32_t stage_words;  // shared-memory words per CTA (set by launch_gselect)
 };
 

@@ -480,7 +480,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (j < nqv) {
                 thr = 0x7FFFFFFFu;
                 if (a.s_sample != nullptr) {
-                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.thr_rank - 1];
                     if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
                 }
             }
@@ -675,7 +675,7 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
             if (j < nqv) {
                 thr = 0x7FFFFFFFu;
                 if (a.s_sample != nullptr) {
-                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.thr_rank - 1];
                     if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
                 }
             }
@@ -862,7 +862,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
             if (j < nqv) {
                 thr = 0x7FFFFFFFu;
                 if (a.s_sample != nullptr) {
-                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.r - 1];
+                    const float s_r = a.s_sample[(int64_t)(q0 + j) * a.r + a.thr_rank - 1];
                     if (s_r > -INFINITY) thr = __float_as_uint(-s_r);
                 }
             }
@@ -1017,8 +1017,32 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
     const bool overflowed = c > (uint64_t)a.cap;
     const int n = overflowed ? (int)a.cap : (int)c;
     if (a.lim_out != nullptr && !overflowed) {
-        // recovery preparation: this list is complete, nothing to redo
-        if (threadIdx.x == 0) a.lim_out[q] = kNoCandidate;
+        // Recovery preparation of a list within its capacity: complete,
+        // unless it holds fewer than r real words after the optimistic
+        // threshold (then every key up to the sample's r-th distance, a safe
+        // bound, is scanned again).
+        bool under = false;
+        if (a.check_underflow) {
+            if (threadIdx.x == 0) sh.nreal = 0;
+            __syncthreads();
+            int real = 0;
+            for (int j = threadIdx.x; j < n; j += kSelThreads) real += list[j] != kNoCandidate;
+            real = __reduce_add_sync(~0u, real);
+            if ((threadIdx.x & 31) == 0) atomicAdd(&sh.nreal, real);
+            __syncthreads();
+            under = sh.nreal < a.r;
+        }
+        if (threadIdx.x == 0) {
+            uint64_t lim = kNoCandidate;
+            if (under) {
+                const float s_r = a.s_sample[(int64_t)q * a.r + a.r - 1];
+                lim = s_r > -INFINITY ? (((uint64_t)__float_as_uint(-s_r) << 32) | 0xFFFFFFFFull)
+                                      : kNoCandidate - 1;  // fewer than r sampled keys: all
+                a.cnt[q] = 0;
+                a.group_flag[q / a.group_size] = 1;
+            }
+            a.lim_out[q] = lim;
+        }
         return;
     }
     if (a.words_out != nullptr && overflowed && threadIdx.x == 0)

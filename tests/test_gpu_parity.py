@@ -537,6 +537,34 @@ def test_wide_batch_list_overflow_is_recovered(nest, B):
             assert out["idx"][b].cpu().numpy().tolist() == copies.tolist()
 
 
+def test_wide_batch_threshold_underflow_is_rescanned(nest):
+    """The main pass of a large batch admits keys up to the sample's j-th
+    distance with j well below r' (here j = 37, r' = 272), expecting about
+    4 r' keys of the datastore below it.  Here every key near the queries
+    sits at a sampled position (400 of them, one every stride-th key), so
+    only 37 keys pass: the list holds fewer than r' words, and the query is
+    scanned again up to the sample's r'-th distance, which is safe.  The
+    result must be the oracle's.  bf16, d=64, N=2,000,000, B=300, r=256."""
+    g = torch.Generator().manual_seed(93)
+    N, d, B, r, vocab = 2_000_000, 64, 300, 256, 300
+    plan = nest.plan_offline(N, d, "bf16", B, r)
+    assert plan["path"] == 3 and not plan["single_pass"]
+    stride = plan["sample_stride"]
+    K = 3.0 + torch.randn(N, d, generator=g)
+    near = torch.arange(0, 400 * stride, stride)
+    K[near] = 0.5 * torch.randn(len(near), d, generator=g)
+    K = K.to(torch.bfloat16)
+    q = (0.1 * torch.randn(B, d, generator=g)).to(torch.bfloat16)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g), dim=1)
+    rows = sorted(set(list(range(0, B, 23)) + [B - 1]))
+    out, _, _ = run_and_check(nest, K, V, q, p_lm, r, 1 / 8, 0.7, vocab, "bf16", check_rows=rows)
+    # every neighbour is one of the near keys
+    near_set = set(near.tolist())
+    for b in rows:
+        assert set(out["idx"][b].cpu().numpy().tolist()) <= near_set
+
+
 @pytest.mark.parametrize("N,d,B,r", [
     (200000, 128, 2048, 64),   # 8 query groups over 19 key ranges, two passes
     (70017, 64, 4000, 33),     # 16 groups (the last one partial), one pass

@@ -45,16 +45,16 @@ def test_decode_plan(nest):
 
 def test_large_batch_plan(nest):
     """B=512, 4M keys, r=256: two groups of 256 queries, every key range once
-    per group in one wave (2 x 76 CTAs), thresholds from every 60th key
-    (about max(65,536, 256 r') sampled keys, r' = 256 + 16 screened
-    candidates kept for the exact re-ranking)."""
-    rp = 256 + 16
+    per group in one wave (2 x 76 CTAs), thresholds from every 64th key
+    (max(65,536, 64 r') sampled keys, r' = 256 + 16 screened candidates kept
+    for the exact re-ranking).  The main pass admits keys up to the sample's
+    32nd distance: about 32 x 64 = 2,048 survivors per query, and the lists
+    hold 8x that."""
     p = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM)
     assert p["kernel"] == "tc_wide2_kernel"
     assert (p["queries_per_group"], p["groups"], p["parts"]) == (256, 2, SMS // 2)
-    assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // (256 * rp)
-    sample = (1 << 22) // p["sample_stride"]
-    assert p["list_capacity"] >= 8 * ((1 << 22) * rp // sample)  # 8x the expected survivors
+    assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // 65536
+    assert p["list_capacity"] >= 8 * 32 * 64  # 8x the expected survivors
     q = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
                           cta_pairs=True)
     assert q["kernel"] == "tc_wide_pair_kernel"
@@ -108,11 +108,12 @@ def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
             if p["single_pass"]:
                 assert p["sample_stride"] == 1 and p["list_capacity"] == N, tag
             else:
-                k = 256 if qpg == 256 else 64
-                target = max(65536, k * r)
+                # r' = r + m screened candidates, m = r / 16 within [16, 128]
+                rp = r + min(128, max(16, r // 16))
+                target = max(65536, 64 * rp)
                 assert p["sample_stride"] == N // target >= 2, tag
                 assert N // p["sample_stride"] >= target, tag
-                assert p["list_capacity"] >= min(N, 8 * r), tag
+                assert p["list_capacity"] >= min(N, 8 * rp), tag
             assert p["scratch_bytes"] >= B * p["list_capacity"] * 8, tag
     assert seen >= {"scan_topr_kernel", "tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
                     "tc_wide_pair_kernel"}, seen
