@@ -352,6 +352,11 @@ def run_reference(args, w, B, world, rank):
 # streams; only valid for the kernel versions captured.  None: not captured
 # for the current kernel.
 TRAFFIC = {
+    # tc_wide2_kernel main pass, d=8192, B=256: a 557,056-key capture; reads x N / 557,056,
+    # survivor writes as they are (about 4 r' per query at any N)
+    ("hidden8192", "tc_wide2_kernel", 256): 9177019648 * 8388608 / 557056 + 35045632,
+    # tc_wide2_kernel main pass, large batch: a 262,144-key capture; reads x16, writes as they are
+    ("large_batch", "tc_wide2_kernel", 512): 2363021056 * 16 + 33024256,
     # tc_scan_kernel<4>, decode: a 65,536-key capture; reads x16, per-CTA list writes as they are
     ("decode", "tc_scan_kernel", 4): 537274880 * 16 + 2926080,
     # tc_scan_kernel<1>, ragged: captured at full size
