@@ -75,11 +75,12 @@ struct SearchPlan {
     ScanPlan scan;
     TcPlan tcp;
     int nq, groups, parts;
+    bool two_phase;      // merge by per-list summaries (merge.cu) instead of a tree
     size_t cand_words;   // scan output: groups * parts * nq * rp
     size_t level_words;  // merge level outputs (ping-pong partner of the scan output)
     size_t cnt_words;    // list lengths of the scan output and of the merge levels
     size_t off_fin;      // each query's rp candidates for the re-ranking: B * rp words,
-                         // B int32 lengths and 3 * B uint32 of re-ranking state (rounded
+                         // B int32 lengths and 2 * B uint32 of re-ranking state (rounded
                          // up to whole words), then B 64-bit words of state
     size_t total_words;  // all scratch of the search
     // Large query batches (tc_wide.cu): sample pass + thresholded pass.
@@ -92,6 +93,7 @@ struct SearchPlan {
     int64_t cap_s, cap_m;     // list capacities per query
     int32_t resv;             // main pass: list slots an epilogue warp reserves at a time
     size_t off_cnt, off_qn, off_lim, off_cand_s, off_s_s, off_i_s, off_cand_m, wide_words;
+    size_t cnt_ints;          // int32 counters and flags zeroed per search
 };
 
 // Parts per query group.  Time ~ waves * (work per part + fixed cost per part),
@@ -131,7 +133,7 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
     const int r = r_out + refine_margin(r_out);
     sp->r = r_out;
     sp->rp = r;
-    const size_t fin_words = (size_t)B * r + ((size_t)4 * B + 1) / 2 + (size_t)B;
+    const size_t fin_words = (size_t)B * r + ((size_t)3 * B + 1) / 2 + (size_t)B;
     sp->tc = false;
     const int64_t keys_per_group_full = ds->N;
     if (ds->tc) {
@@ -178,6 +180,8 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
     const int per = merge_fanin(sp->parts, r);
     const int lvl1 = (sp->parts + per - 1) / per;
     sp->level_words = lvl1 > 1 ? (size_t)B * lvl1 * r : 0;
+    sp->two_phase = merge_two_phase(sp->parts, r);
+    if (sp->two_phase) sp->level_words = merge_two_phase_words(B, sp->parts);
     // int32 counts: [groups * parts * nq] then [B * lvl1], as 64-bit words
     sp->cnt_words = ((size_t)sp->groups * sp->parts * sp->nq + 1) / 2 + ((size_t)B * lvl1 + 1) / 2;
     sp->off_fin = sp->cand_words + sp->level_words + sp->cnt_words;
@@ -237,8 +241,10 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
             sp->wpr.groups = wp.groups;
             sp->wpr.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
             // 2 * B int32 counters, then kRecoverRounds * groups int32 flags
+            // (zeroed by one memset per search)
             sp->off_cnt = 0;
-            sp->off_qn = (2 * (size_t)B + (size_t)kRecoverRounds * wp.groups + 1) / 2;
+            sp->cnt_ints = 2 * (size_t)B + (size_t)kRecoverRounds * wp.groups;
+            sp->off_qn = (sp->cnt_ints + 1) / 2;
             sp->off_lim = sp->off_qn + ((size_t)B + 1) / 2;  // after B floats ||q||^2
             sp->off_cand_s = sp->off_lim + (size_t)B;       // after B word limits
             sp->off_s_s = sp->off_cand_s + (size_t)B * sp->cap_s;
@@ -457,8 +463,7 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     nest_status_t st;
     int32_t* cnt = reinterpret_cast<int32_t*>(scratch + sp.off_cnt);
     int32_t* flags = cnt + 2 * (size_t)B;  // kRecoverRounds rows of groups
-    cudaError_t e = cudaMemsetAsync(
-        cnt, 0, sizeof(int32_t) * (2 * (size_t)B + (size_t)kRecoverRounds * sp.wpm.groups), stream);
+    cudaError_t e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * sp.cnt_ints, stream);
     if (e != cudaSuccess) return from_cuda(e);
     CUtensorMap qmap;
     // a CTA of a pair stages half of the group's queries
@@ -614,7 +619,7 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
     uint64_t* fin = scratch + sp.off_fin;
     int32_t* fin_cnt = reinterpret_cast<int32_t*>(fin + (size_t)B * r);
     uint32_t* state = reinterpret_cast<uint32_t*>(fin_cnt + B);
-    auto* apair = reinterpret_cast<unsigned long long*>(fin + (size_t)B * r + (4 * (size_t)B + 1) / 2);
+    auto* apair = reinterpret_cast<unsigned long long*>(fin + (size_t)B * r + (3 * (size_t)B + 1) / 2);
 
     cudaError_t e;
     if (sp.wide) {
@@ -683,7 +688,19 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
         ma.B = B;
         ma.r = r;
         bool into_b = true;
-        for (;;) {
+        if (sp.two_phase) {
+            // per-list summaries (their largest words first, then the words)
+            ma.tsum = regionB;
+            ma.sum = regionB + (size_t)B * sp.parts;
+            ma.out = fin;
+            ma.out_cnt = fin_cnt;
+            ma.refine_state = state;
+            ma.refine_apair = apair;
+            e = launch_merge_two_phase(ma, stream);
+            if (e != cudaSuccess) return from_cuda(e);
+            ds->launches += 2;
+        }
+        for (; !sp.two_phase;) {
             ma.per_cta = merge_fanin(ma.lists, r);
             const int groups = (ma.lists + ma.per_cta - 1) / ma.per_cta;
             const bool last = groups == 1;

@@ -251,6 +251,9 @@ struct MergeArgs {
     int32_t* out_cnt;      // [B][ceil(lists / per_cta)] real entries of each output list
     uint32_t* refine_state;  // non-null on the final level (one list per query): the exact
     unsigned long long* refine_apair;  // re-ranking's state is reset for each query
+    // two-phase merge only: [B][lists][32] summary words and [B][lists] their largest
+    uint64_t* sum;
+    uint64_t* tsum;
 };
 
 int merge_lists_per_cta(int r);
@@ -258,23 +261,27 @@ int merge_lists_per_cta(int r);
 int merge_fanin(int lists, int r);
 size_t merge_smem_bytes(int per_cta, int r);
 cudaError_t launch_merge(const MergeArgs& args, cudaStream_t stream);
+// Whether the two-phase merge (per-list summaries, then one CTA per query)
+// applies to `lists` lists of up to r words per query, the scratch words its
+// summaries take, and its two launches (out / out_cnt: one list per query).
+bool merge_two_phase(int lists, int r);
+size_t merge_two_phase_words(int B, int lists);
+cudaError_t launch_merge_two_phase(const MergeArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- refine.cu
 // Exact re-ranking: each query's r' = r + refine_margin(r) screened
 // candidates get their distances recomputed as sums of squared differences;
 // the r nearest by those are sorted into s and idx.
 //
-// Per-query state: three rows of B 32-bit words (CTAs finished, largest and
-// smallest screening error as fp32 ordered bits) and B 64-bit words (the
-// largest screened distance's bits above its candidate's exact distance
-// bits).  The kernel that writes a query's candidate list resets the
-// query's entries.
+// Per-query state: two rows of B 32-bit words (largest and smallest
+// screening error as fp32 ordered bits) and B 64-bit words (the largest
+// screened distance's bits above its candidate's exact distance bits).  The
+// kernel that writes a query's candidate list resets the query's entries.
 __device__ __forceinline__ void refine_state_reset(uint32_t* state, unsigned long long* apair,
                                                    int B, int b)
 {
     state[b] = 0;
-    state[B + b] = 0;
-    state[2 * B + b] = ~0u;
+    state[B + b] = ~0u;
     apair[b] = 0;
 }
 
@@ -284,7 +291,7 @@ struct RefineArgs {
     int32_t row_bytes;   // d * element size
     uint64_t* cand;      // [B][rp] screened words (distance bits : key), rewritten in place
     const int32_t* cand_cnt;  // [B] real words of each list
-    uint32_t* state;     // [3][B], reset by the kernel that wrote the lists
+    uint32_t* state;     // [2][B], reset by the kernel that wrote the lists
     unsigned long long* apair;  // [B], likewise
     int* status;
     int32_t B;

@@ -11,14 +11,23 @@
 // squared differences of the stored elements (fp32, exact products of the
 // widened bf16 values; eight interleaved partial sums per lane and a warp
 // tree, so at most ~40 additions separate any term from the result).  It
-// then keeps the r nearest by those distances (ties: smaller key index),
-// sorts them and writes s = -distance and the key index.
+// then puts the r nearest by those distances in order (ties: smaller key
+// index) and writes s = -distance and the key index.
 //
-// Grid (chunks of 16 candidates, B queries), 512 threads: warp w of chunk c
-// recomputes candidate 16 c + w, eight 16-byte loads in flight per lane.  A
-// CTA rewrites its candidates' words in place, and the last CTA of a query
-// to finish (an atomic counter, no wait) sorts the r' words (bitonic, in
-// shared memory) and writes the first r.
+// Two kernels (the second a programmatic dependent of the first):
+//   refine_dist_kernel  grid (chunks of 16 candidates, B queries), 512
+//                       threads: warp w of chunk c recomputes candidate
+//                       16 c + w, all of its row's 16-byte loads in flight
+//                       at once (8 or 16 KiB rows), and rewrites the word in
+//                       place; each CTA folds its screening errors into the
+//                       query's state with atomics.
+//   refine_rank_kernel  grid (chunks of 16 candidates, B queries), 512
+//                       threads: warp w of chunk c takes candidate 16 c + w,
+//                       counts the query's words below its own (the words
+//                       are distinct, so the counts are the sorted
+//                       positions), and writes s and idx at that position
+//                       when it is below r.  No sort and no CTA that waits
+//                       for the others.
 //
 // It also checks the margin.  A key left out of the r' candidates had a
 // screened distance of at least A, the largest screened distance kept.  The
@@ -38,14 +47,14 @@
 
 #include "internal.h"
 #include "ptx.cuh"
-#include "select.cuh"
 
 namespace nest {
 namespace {
 
 constexpr int kRefineThreads = 512;
 constexpr int kRefineRows = kRefineThreads / 32;  // candidates per CTA
-constexpr int kRefineLoads = 8;                   // 16-byte loads in flight per lane
+constexpr int kRefineLoads = 16;                  // 16-byte loads in flight per lane
+constexpr int kRankThreads = 512;  // one warp per position, 16 per CTA
 // Distance bits no real distance has (a NaN pattern above +inf's bits).
 constexpr uint64_t kPadHigh = 0xFFFFFFFFull << 32;
 
@@ -63,15 +72,7 @@ __device__ __forceinline__ float from_ordered_bits(uint32_t o)
 struct RefineShared {
     uint32_t emax, emin;      // largest / smallest screened - exact distance (ordered bits)
     unsigned long long apair; // largest (screened bits << 32 | exact bits) of this CTA
-    int last;
 };
-
-__host__ __device__ inline int pow2_at_least(int x)
-{
-    int p = 1;
-    while (p < x) p <<= 1;
-    return p;
-}
 
 // Sum of squared differences of one 16-byte chunk (8 bf16 or 4 fp32 values)
 // into the lane's partial sums.
@@ -98,11 +99,10 @@ __device__ __forceinline__ void chunk_sqdiff(const uint4& k, const uint4& q, flo
 }
 
 template <int DT>
-__global__ void __launch_bounds__(kRefineThreads) refine_kernel(const RefineArgs a)
+__global__ void __launch_bounds__(kRefineThreads) refine_dist_kernel(const RefineArgs a)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     uint4* qs = reinterpret_cast<uint4*>(smem);  // the query row
-    uint64_t* buf = reinterpret_cast<uint64_t*>(smem + a.row_bytes);
     __shared__ RefineShared sh;
     grid_dependency_wait();
     grid_dependents_launch();
@@ -111,6 +111,8 @@ __global__ void __launch_bounds__(kRefineThreads) refine_kernel(const RefineArgs
     const int chunks = a.row_bytes / 16;
     uint64_t* list = a.cand + (int64_t)b * a.rp;
     const int n = min(max(a.cand_cnt[b], 0), a.rp);
+    const int j = blockIdx.x * kRefineRows + warp;
+    const uint64_t w = j < n ? list[j] : kNoCandidate;
 
     const uint4* qrow = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(a.q) +
                                                        (size_t)b * a.row_bytes);
@@ -123,91 +125,94 @@ __global__ void __launch_bounds__(kRefineThreads) refine_kernel(const RefineArgs
     __syncthreads();
 
     // ---- one warp per candidate: exact distance, word rewritten in place
-    const int j = blockIdx.x * kRefineRows + warp;
-    if (j < n) {
-        const uint64_t w = list[j];
-        if (w != kNoCandidate) {
-            const uint32_t key = (uint32_t)w;
-            const uint4* krow = reinterpret_cast<const uint4*>(
-                static_cast<const unsigned char*>(a.K) + (size_t)key * a.row_bytes);
-            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            int c = lane;
-            for (; c + (kRefineLoads - 1) * 32 < chunks; c += kRefineLoads * 32) {
-                uint4 kv[kRefineLoads];
+    if (w != kNoCandidate) {
+        const uint32_t key = (uint32_t)w;
+        const uint4* krow = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(a.K) +
+                                                           (size_t)key * a.row_bytes);
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        int c = lane;
+        for (; c + (kRefineLoads - 1) * 32 < chunks; c += kRefineLoads * 32) {
+            uint4 kv[kRefineLoads];
 #pragma unroll
-                for (int u = 0; u < kRefineLoads; ++u) kv[u] = ld_global_nc_v4(krow + c + 32 * u);
+            for (int u = 0; u < kRefineLoads; ++u) kv[u] = ld_global_nc_v4(krow + c + 32 * u);
+            // every load is issued before the first use of any: the empty
+            // volatile statements keep the arithmetic after all sixteen
 #pragma unroll
-                for (int u = 0; u < kRefineLoads; ++u) chunk_sqdiff<DT>(kv[u], qs[c + 32 * u], acc);
-            }
-            for (; c < chunks; c += 32) chunk_sqdiff<DT>(ld_global_nc_v4(krow + c), qs[c], acc);
-            float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+            for (int u = 0; u < kRefineLoads; ++u)
+                asm volatile("" : "+r"(kv[u].x), "+r"(kv[u].y), "+r"(kv[u].z), "+r"(kv[u].w));
 #pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
-            if (lane == 0) {
-                const float screened = __uint_as_float((uint32_t)(w >> 32));
-                list[j] = ((uint64_t)__float_as_uint(s) << 32) | key;
-                __threadfence();  // the word is visible before this CTA counts itself done
-                const uint32_t e = ordered_bits(screened - s);
-                atomicMax(&sh.emax, e);
-                atomicMin(&sh.emin, e);
-                // distances are >= 0, so their bits order like the values
-                atomicMax(&sh.apair, ((unsigned long long)(w >> 32) << 32) | __float_as_uint(s));
-            }
+            for (int u = 0; u < kRefineLoads; ++u) chunk_sqdiff<DT>(kv[u], qs[c + 32 * u], acc);
+        }
+        for (; c < chunks; c += 32) chunk_sqdiff<DT>(ld_global_nc_v4(krow + c), qs[c], acc);
+        float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) s += __shfl_xor_sync(~0u, s, o);
+        if (lane == 0) {
+            const float screened = __uint_as_float((uint32_t)(w >> 32));
+            list[j] = ((uint64_t)__float_as_uint(s) << 32) | key;
+            const uint32_t e = ordered_bits(screened - s);
+            atomicMax(&sh.emax, e);
+            atomicMin(&sh.emin, e);
+            // distances are >= 0, so their bits order like the values
+            atomicMax(&sh.apair, ((unsigned long long)(w >> 32) << 32) | __float_as_uint(s));
         }
     }
     __syncthreads();
-    if (tid == 0) {
-        atomicMax(&a.state[a.B + b], sh.emax);
-        atomicMin(&a.state[2 * a.B + b], sh.emin);
+    if (tid == 0 && sh.emin != ~0u) {
+        atomicMax(&a.state[b], sh.emax);
+        atomicMin(&a.state[a.B + b], sh.emin);
         atomicMax(&a.apair[b], sh.apair);
-        __threadfence();
-        const uint32_t prev = atomicAdd(&a.state[b], 1u);
-        sh.last = prev == gridDim.x - 1;
     }
-    __syncthreads();
-    if (!sh.last) return;
-    __threadfence();
+}
 
-    // ---- last CTA of this query: all candidates sorted by exact distance
-    // (ties: smaller key index), the first r written.  A padding word (none
-    // is expected among the n) becomes a distinct word above every real one.
-    const int P2 = pow2_at_least(n > 0 ? n : 1);
-    for (int i = tid; i < P2; i += kRefineThreads) {
-        uint64_t w = kNoCandidate;
-        if (i < n) {
-            w = __ldcg(list + i);
-            if (w == kNoCandidate) w = kPadHigh | (uint32_t)i;
-        }
-        buf[i] = w;
+__global__ void __launch_bounds__(kRankThreads) refine_rank_kernel(const RefineArgs a)
+{
+    extern __shared__ __align__(16) uint64_t words[];  // the query's n words
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int b = blockIdx.y;
+    const uint64_t* list = a.cand + (int64_t)b * a.rp;
+    const int n = min(max(a.cand_cnt[b], 0), a.rp);
+    // A padding word (none is expected among the n) becomes a distinct
+    // word above every real one, so the positions stay a permutation.
+    for (int i = tid; i < n; i += kRankThreads) {
+        const uint64_t w = list[i];
+        words[i] = w != kNoCandidate ? w : (kPadHigh | (uint32_t)i);
     }
     __syncthreads();
-    bitonic_sort<kRefineThreads>(buf, P2, tid, [] { __syncthreads(); });
-    const int m = n < a.r ? n : a.r;
+    // one warp per position i: candidate i's rank, or the padding of a short row
+    const int i = blockIdx.x * (kRankThreads / 32) + warp;
     float* so = a.s_out + (int64_t)b * a.r;
     int64_t* io = a.idx_out + (int64_t)b * a.r;
-    for (int i = tid; i < a.r; i += kRefineThreads) {
-        const uint64_t e = i < m ? buf[i] : kNoCandidate;
-        if ((e >> 32) < 0xFFFFFFFFu) {
-            so[i] = -__uint_as_float((uint32_t)(e >> 32));
-            io[i] = (int64_t)(uint32_t)e;
-        } else {
-            so[i] = -INFINITY;
-            io[i] = -1;
+    if (i < n) {
+        const uint64_t mine = words[i];
+        int below = 0;
+        for (int k = lane; k < n; k += 32) below += words[k] < mine;
+        const int rank = __reduce_add_sync(~0u, below);
+        if (lane == 0 && rank < a.r) {
+            if ((mine >> 32) < 0xFFFFFFFFu) {
+                so[rank] = -__uint_as_float((uint32_t)(mine >> 32));
+                io[rank] = (int64_t)(uint32_t)mine;
+            } else {
+                so[rank] = -INFINITY;
+                io[rank] = -1;
+            }
         }
-    }
-    if (tid == 0) {
-        // Keys outside the candidates exist only when the list is full.
-        if (n == a.rp && m == a.r) {
-            const float A_exact = __uint_as_float((uint32_t)__ldcg(&a.apair[b]));
-            const float emax = from_ordered_bits(__ldcg(&a.state[a.B + b]));
-            const float emin = from_ordered_bits(__ldcg(&a.state[2 * a.B + b]));
-            const float Dr = __uint_as_float((uint32_t)(buf[a.r - 1] >> 32));
+        if (lane == 0 && rank == a.r - 1 && n == a.rp) {
+            // The margin (keys outside the candidates exist only when the
+            // list is full); the kernel that writes the lists resets the state.
+            const float A_exact = __uint_as_float((uint32_t)a.apair[b]);
+            const float emax = from_ordered_bits(a.state[b]);
+            const float emin = from_ordered_bits(a.state[a.B + b]);
+            const float Dr = __uint_as_float((uint32_t)(mine >> 32));
             const float W = 2.f * (emax - emin);
             const bool ok = (A_exact - W > Dr) || (A_exact == Dr);
             if (!ok) record_status(a.status, NEST_ERR_MARGIN);
         }
-        // ready for the next search (the kernel before this one also resets them)
-        refine_state_reset(a.state, a.apair, a.B, b);
+    } else if (i < a.r && lane == 0) {
+        so[i] = -INFINITY;  // positions n .. r - 1 of a short row
+        io[i] = -1;
     }
 }
 
@@ -222,21 +227,32 @@ int refine_margin(int r)
 size_t refine_smem_bytes(int rp, int r, int row_bytes)
 {
     (void)r;
-    return (size_t)row_bytes + (size_t)pow2_at_least(rp) * sizeof(uint64_t);
+    const size_t words = (size_t)rp * sizeof(uint64_t);
+    return words > (size_t)row_bytes ? words : (size_t)row_bytes;
 }
 
 cudaError_t launch_refine(int dtype, const RefineArgs& a, cudaStream_t stream)
 {
     const dim3 grid((a.rp + kRefineRows - 1) / kRefineRows, a.B);
-    const size_t smem = refine_smem_bytes(a.rp, a.r, a.row_bytes);
+    const size_t qbytes = (size_t)a.row_bytes;
+    cudaError_t e;
     if (dtype == NEST_BF16) {
-        cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(refine_kernel<NEST_BF16>), smem);
-        if (e != cudaSuccess) return e;
-        return launch_pdl(refine_kernel<NEST_BF16>, grid, dim3(kRefineThreads), smem, stream, a);
+        e = raise_smem_limit(reinterpret_cast<const void*>(refine_dist_kernel<NEST_BF16>), qbytes);
+        if (e == cudaSuccess)
+            e = launch_pdl(refine_dist_kernel<NEST_BF16>, grid, dim3(kRefineThreads), qbytes, stream, a);
+    } else {
+        e = raise_smem_limit(reinterpret_cast<const void*>(refine_dist_kernel<NEST_F32>), qbytes);
+        if (e == cudaSuccess)
+            e = launch_pdl(refine_dist_kernel<NEST_F32>, grid, dim3(kRefineThreads), qbytes, stream, a);
     }
-    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(refine_kernel<NEST_F32>), smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(refine_kernel<NEST_F32>, grid, dim3(kRefineThreads), smem, stream, a);
+    // rank threads cover max(r', r) positions: candidates, then the padding of short rows
+    const int cover = a.rp > a.r ? a.rp : a.r;
+    const dim3 rgrid((cover + kRankThreads / 32 - 1) / (kRankThreads / 32), a.B);
+    const size_t wbytes = (size_t)a.rp * sizeof(uint64_t);
+    e = raise_smem_limit(reinterpret_cast<const void*>(refine_rank_kernel), wbytes);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(refine_rank_kernel, rgrid, dim3(kRankThreads), wbytes, stream, a);
 }
 
 }  // namespace nest

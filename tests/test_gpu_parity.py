@@ -167,6 +167,28 @@ def test_key_equal_to_query_is_first_with_distance_zero(nest):
     assert out["idx"][:, 0].cpu().tolist() == [17, 9999, 4242]
 
 
+@pytest.mark.parametrize("r", [1024, 4096])
+def test_narrow_scan_keys_stored_cluster_by_cluster(nest, r):
+    """Keys stored cluster after cluster: a query's nearest keys all sit in
+    the two or three key ranges that hold its cluster, so those ranges'
+    candidate lists hold far more of the r' nearest than their 32-word
+    summaries, and the two-phase merge must read them whole (r = 1024: in
+    shared memory at once; r = 4096: more than it holds, one list at a time).
+    bf16, d=128, N=200,000 in 64 contiguous clusters, B=4."""
+    N, d, B, vocab = 200000, 128, 4, 500
+    g = torch.Generator().manual_seed(61 + r)
+    c = torch.randn(64, d, generator=g)
+    assign = torch.arange(N) // (N // 64)
+    assign.clamp_(max=63)
+    K = (c[assign] + 0.3 * torch.randn(N, d, generator=g)).to(torch.bfloat16)
+    q = (c[torch.tensor([5, 5, 40, 63])] + 0.3 * torch.randn(B, d, generator=g)).to(torch.bfloat16)
+    V = torch.randint(0, vocab, (N,), generator=g, dtype=torch.int32)
+    p_lm = torch.softmax(torch.randn(B, vocab, generator=g), dim=1)
+    plan = nest.plan_offline(N, d, "bf16", B, r)
+    assert plan["path"] == 1 and plan["parts"] >= 64, plan
+    run_and_check(nest, K, V, q, p_lm, r, 1 / np.sqrt(d), 0.7, vocab, "bf16")
+
+
 def test_margin_check_reports_a_crowded_boundary(nest):
     """Keys whose exact distances are packed closer than the fp32 screening
     error: integer vectors of about 1,000-norm-squared per element (||q||^2 and
