@@ -64,9 +64,10 @@ def parse():
                    help="knnlm: search + Eq. 2 + Eq. 3 (default); nest: masked search + Eq. 2 + "
                         "Eq. 4 + Eq. 5/6 decision; verify: a batch of drafted positions "
                         "searched, mixed (Eq. 4) and verified (Eq. 7)")
-    p.add_argument("--cta-pairs", action="store_true",
-                   help="run groups of 256 queries on CTA pairs (nest_datastore_use_cta_pairs) "
-                        "instead of the default two-tile kernel")
+    p.add_argument("--cta-pairs", choices=["auto", "on", "off"], default="auto",
+                   help="groups of 256 queries on CTA pairs (nest_datastore_use_cta_pairs): "
+                        "auto (the default: pairs for one group), on, or off (single CTAs "
+                        "with two key tiles per stage)")
     p.add_argument("--sweep", default=None,
                    help="comma-separated query batch sizes measured on one datastore, one JSON "
                         "line each (e.g. 1,8,64,256 for the d=8192 workload)")
@@ -352,8 +353,10 @@ def run_reference(args, w, B, world, rank):
 # streams; only valid for the kernel versions captured.  None: not captured
 # for the current kernel.
 TRAFFIC = {
-    # tc_wide2_kernel main pass, d=8192, B=256: a 557,056-key capture; reads x N / 557,056,
-    # survivor writes as they are (about 4 r' per query at any N)
+    # tc_wide_pair_kernel main pass, d=8192, B=256 (the default for one group): a 557,056-key
+    # capture; reads x N / 557,056, survivor writes as they are (about 4 r' per query at any N)
+    ("hidden8192", "tc_wide_pair_kernel", 256): 9239347456 * 8388608 / 557056 + 79070208,
+    # tc_wide2_kernel main pass, same workload on single CTAs (--cta-pairs off)
     ("hidden8192", "tc_wide2_kernel", 256): 9177019648 * 8388608 / 557056 + 35045632,
     # tc_wide2_kernel main pass, large batch: a 262,144-key capture; reads x16, writes as they are
     ("large_batch", "tc_wide2_kernel", 512): 2363021056 * 16 + 33024256,
@@ -418,8 +421,7 @@ def main():
     B_gen = max(b for b in sweep if b is not None) if any(b is not None for b in sweep) else None
     x = synth.make_inputs(w, device=dev, B=B_gen, N=args.N, seed=w.seed + rank)
     ds = nest.Datastore(x.K, x.V, w.vocab)
-    if args.cta_pairs:
-        ds.use_cta_pairs(True)
+    ds.use_cta_pairs({"auto": None, "on": True, "off": False}[args.cta_pairs])
     lines = []
     for B in sweep:
         lines.append(measure(args, w, x, ds, B if B is not None else x.q.shape[0], world, rank,

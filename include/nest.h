@@ -107,21 +107,30 @@ NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_
                                      int32_t ragged);
 
 /*
- * Whether searches with groups of 256 queries run on CTA pairs (search
- * path 4 of nest_search_path) or on single CTAs with two key tiles per
- * pipeline stage (path 3, the default).  Both return the same neighbours.
- * A pair splits each 256-key tile over two SMs and double-buffers its
- * accumulators; with one query group it runs as fast as path 3, but with
- * several groups their pairs drift apart and read the same keys from DRAM
- * again (1.20 times the key bytes at 1M keys and B = 512 on a GB300,
- * against 1.09 for path 3), so path 3 stays the default.  Pairs need two
- * CTAs of about 220 KiB of shared memory each on the two SMs of one TPC at
- * the same time; on = 1 where the device cannot place them returns
- * NEST_ERR_UNSUPPORTED and changes nothing.  Host only; takes effect from
- * the next search, which may need more scratch than nest_datastore_reserve
- * set aside.
+ * How searches with groups of 256 queries are laid out on the SMs (search
+ * paths 3 and 4 of nest_search_path).  Both return the same neighbours.
+ *
+ *   mode  1  always on CTA pairs (path 4): each 256-key tile is split over
+ *            the two SMs of a pair and each CTA stages only half of the
+ *            group's queries, so a pipeline stage carries the MMA work of a
+ *            path-3 stage in three quarters of the shared memory (four
+ *            stages instead of three).
+ *   mode  0  never: single CTAs with two 128-key tiles per stage (path 3).
+ *   mode -1  automatic, the default: pairs when the batch is one group
+ *            (129 to 256 queries), single CTAs for more groups.  With one
+ *            group the pairs' main pass is about 4 % faster (d = 8192,
+ *            8M keys, B = 256 on a GB300); with several groups their pairs
+ *            drift apart over the same keys and read them from DRAM again,
+ *            which made them about 5 % slower (4M keys, B = 512).
+ *
+ * Pairs need two CTAs of about 220 KiB of shared memory each on the two SMs
+ * of one TPC at the same time; mode 1 where the device cannot place them
+ * returns NEST_ERR_UNSUPPORTED and changes nothing, and mode -1 there runs
+ * single CTAs.  Any other mode returns NEST_ERR_INVALID_ARG.  Host only;
+ * takes effect from the next search, which may need more scratch than
+ * nest_datastore_reserve set aside.
  */
-NEST_API nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t on);
+NEST_API nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t mode);
 
 /*
  * r-nearest-neighbour search (Sec. 2.2; Sec. 3.1 second stage; App. A).
@@ -377,8 +386,8 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
  *   3  the same with two 128-key tiles per pipeline stage (groups of 256
  *      queries, when three 64 KiB stages fit in shared memory)
  *   4  the same on CTA pairs (groups of 256 queries, 256-key tiles split
- *      over two SMs, double-buffered accumulators), after
- *      nest_datastore_use_cta_pairs(ds, 1)
+ *      over two SMs, two such tiles per stage): by default when the batch
+ *      is one group; see nest_datastore_use_cta_pairs
  * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
  */
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,
@@ -391,8 +400,8 @@ NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t
  * nest_knn_search on a datastore of N keys of d elements of `dtype`, on a
  * device with `num_sms` SMs and `smem_per_block` bytes of opt-in shared
  * memory per block (cudaDevAttrMaxSharedMemoryPerBlockOptin), with
- * nest_datastore_use_cta_pairs(ds, cta_pairs) in effect (the device is
- * assumed able to place the pairs).  Arguments are checked as
+ * nest_datastore_use_cta_pairs(ds, cta_pairs) in effect (1, 0 or -1, the
+ * handle's default; the device is assumed able to place the pairs).  Arguments are checked as
  * nest_datastore_create and nest_knn_search check them.
  */
 typedef struct nest_plan {
@@ -422,7 +431,8 @@ NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
 NEST_API const char* nest_status_string(nest_status_t status);
 
 /* ABI version: major * 10000 + minor * 100 + patch (0.2.0: CTA pairs and
- * the bounded-wait self-test added to 0.1.0). */
+ * the bounded-wait self-test added to 0.1.0; 0.3.0: CTA pairs with two
+ * 256-key tiles per stage, chosen automatically for one query group). */
 NEST_API int32_t nest_version(void);
 
 #ifdef __cplusplus

@@ -28,7 +28,7 @@ struct nest_datastore {
     size_t smem_optin = 0;
     bool tc = false;         // bf16 keys with a TMA tensor map: tensor-core scan
     bool pairs_ok = false;   // the device can place the wide kernel's CTA pairs
-    bool pairs = false;      // ... and searches use them
+    int pairs_mode = 0;      // 1: groups of 256 on pairs, 0: never, -1: when one group
     CUtensorMap keys_map;  // TMA map of K (type is 64-byte aligned)
     float* knorm = nullptr;  // owned: ||k_i||^2, N floats
     int* status = nullptr;   // owned: device status word
@@ -192,7 +192,12 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
     if (sp->tc && !ragged && sp->groups > 1) {
         const int nm = B >= 256 ? 256 : std::max(16, ceil_pow2(B));
         WidePlan wp{};
-        if (wide_plan_smem(nm, ds->smem_optin, ds->pairs, &wp)) {
+        // CTA pairs: when asked for, or (automatic) when the batch is one
+        // group, whose key ranges no other group's CTAs stream beside them
+        const bool one_group = B <= nm;
+        const bool pairs =
+            ds->pairs_ok && (ds->pairs_mode == 1 || (ds->pairs_mode < 0 && one_group));
+        if (wide_plan_smem(nm, ds->smem_optin, pairs, &wp)) {
             wp.groups = (B + nm - 1) / nm;
             // A sample of every stride-th key, about max(65,536, 64 r) keys.
             const int64_t target = std::max<int64_t>(65536, 64 * (int64_t)r);
@@ -225,8 +230,9 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
             // distance, so a warp that drains `rows` key rows admits about
             // rows * j / sample_rows keys per query; it reserves twice that
             // plus 16 slots at a time (one atomic per block).  Each column
-            // has 4 reserving warps per CTA (8 with two key tiles per stage).
-            const int epi_warps = wp.mb == 2 ? 8 : 4;
+            // has 4 reserving warps per 128-key tile of a step (8 with two
+            // key tiles per stage, 16 over a CTA pair's four).
+            const int epi_warps = 4 * wp.mb;
             const int64_t unit = (int64_t)kTcTileKeys * wp.mb;
             const int64_t units = (ds->N + unit - 1) / unit;
             const int64_t rows = (units + sp->wpm.parts - 1) / sp->wpm.parts * 32;
@@ -841,7 +847,7 @@ nest_status_t nest_datastore_create(const void* K, const int32_t* V, int64_t N, 
     if (dtype == NEST_BF16 && N <= (int64_t)0x7FFFFF00)
         ds->tc = encode_bf16_rows(&ds->keys_map, K, N, d, kTcTileKeys, true);
     ds->pairs_ok = ds->tc && wide_pair_clusters(ds->smem_optin) > 0;
-    ds->pairs = false;  // opt-in: nest_datastore_use_cta_pairs
+    ds->pairs_mode = -1;  // automatic: nest_datastore_use_cta_pairs
     if (host_status != 0) {
         nest_datastore_destroy(ds);
         return static_cast<nest_status_t>(host_status);
@@ -886,11 +892,11 @@ nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_B, int32_
     return ensure_scratch(ds, need);
 }
 
-nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t on)
+nest_status_t nest_datastore_use_cta_pairs(nest_datastore_t* ds, int32_t mode)
 {
-    if (!ds) return NEST_ERR_INVALID_ARG;
-    if (on && !ds->pairs_ok) return NEST_ERR_UNSUPPORTED;
-    ds->pairs = on != 0;
+    if (!ds || mode < -1 || mode > 1) return NEST_ERR_INVALID_ARG;
+    if (mode == 1 && !ds->pairs_ok) return NEST_ERR_UNSUPPORTED;
+    ds->pairs_mode = mode;
     return NEST_OK;
 }
 
@@ -1179,8 +1185,9 @@ nest_status_t nest_plan_offline(int64_t N, int32_t d, nest_dtype_t dtype, int32_
     ds.smem_optin = (size_t)smem_per_block;
     // the key tensor map encodes for every such bf16 datastore (16-byte rows)
     ds.tc = dtype == NEST_BF16 && N <= (int64_t)0x7FFFFF00;
+    if (cta_pairs < -1 || cta_pairs > 1) return NEST_ERR_INVALID_ARG;
     ds.pairs_ok = ds.tc;
-    ds.pairs = ds.tc && cta_pairs != 0;
+    ds.pairs_mode = cta_pairs;
     SearchPlan sp;
     const nest_status_t st = plan_search(&ds, B, r, ragged != 0, &sp);
     if (st != NEST_OK) return st;
@@ -1233,7 +1240,7 @@ const char* nest_status_string(nest_status_t s)
     return "unknown status";
 }
 
-int32_t nest_version(void) { return 200; }
+int32_t nest_version(void) { return 300; }
 
 }  // extern "C"
 

@@ -145,8 +145,9 @@ cudaError_t launch_tc_scan(const TcPlan& plan, const CUtensorMap& keys, const CU
 // Large query batches: threshold-admission scan into global lists + exact selection.
 struct WidePlan {
     int nm;       // MMA N = queries per CTA (16, 32, 64, 128 or 256)
-    int mb;       // 128-key tiles per pipeline stage (2 only for nm = 256)
-    bool pair;    // nm = 256 on CTA pairs (tcgen05 cta_group::2): 256 keys per tile,
+    int mb;       // 128-key tiles per pipeline step: 1, 2 (nm = 256 on one CTA) or 4
+                  // (nm = 256 on a CTA pair: two 256-key tiles)
+    bool pair;    // nm = 256 on CTA pairs (tcgen05 cta_group::2): M = 256 keys per MMA,
                   // each part is a pair of CTAs
     int stages;
     int groups;   // query groups of nm

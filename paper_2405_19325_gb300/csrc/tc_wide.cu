@@ -13,9 +13,9 @@
 //      queries with tcgen05.mma (M = 128 keys, N = up to 256 queries,
 //      K = 16): tc_wide_kernel keeps one key tile per stage and two TMEM
 //      accumulators of N columns.  Groups of 256 run on tc_wide2_kernel
-//      (two key tiles per stage, one accumulator each) or, when asked for,
-//      on CTA pairs (tc_wide_pair_kernel: M = 256 keys over the pair, two
-//      accumulators).  The epilogue warps form
+//      (two key tiles per stage, one accumulator each) or on CTA pairs
+//      (tc_wide_pair_kernel: M = 256 keys over the pair, two such tiles per
+//      stage; the default when the batch is one group).  The epilogue warps form
 //      ||q||^2 + ||k||^2 - 2 q.k, admit the keys under each query's threshold
 //      and append them to that query's global list through per-warp slot
 //      reservations.
@@ -722,31 +722,35 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
 // Groups of 256 queries on CTA pairs (a cluster of two CTAs on one TPC):
 // tcgen05.mma.cta_group::2 with M = 256 keys (128 in each CTA's shared
 // memory and TMEM lanes), N = 256 queries (each CTA stages 128 of them; the
-// MMA reads both halves) and K = 16.  A stage is 16 KiB of keys and 16 KiB
-// of queries per CTA, and TMEM holds two 256-column accumulators, so the
-// epilogue of one 256-key tile overlaps the MMAs of the next (the two-tile
-// kernel above cannot double-buffer: its two tiles fill TMEM).
+// MMA reads both halves) and K = 16, two such 256-key tiles per stage.  Per
+// CTA a stage is 32 KiB of keys and 16 KiB of queries, where the two-tile
+// kernel above stages 32 KiB of keys and the whole 32 KiB query chunk for
+// the same MMA work per SM: the pair reads half as many query bytes from L2
+// and four 48 KiB stages fit where three 64 KiB stages did, so the ring
+// covers a third more latency.  Each CTA's two 256-column accumulators fill
+// its TMEM, so, as in the two-tile kernel, a tile pair's epilogue runs
+// between its last MMA and the next pair's first.
 //   * both CTAs' TMA loads complete on the even CTA's full barrier, which the
 //     even CTA arms with the pair's bytes; the even CTA's MMA thread issues
 //     for the pair and its commits arrive on both CTAs' empty and acc_full
 //     barriers;
-//   * both CTAs' epilogue threads hand the accumulators back on the even
-//     CTA's acc_empty barrier;
+//   * both CTAs' sixteen epilogue warps hand the accumulators back on the
+//     even CTA's acc_empty barrier;
 //   * neither CTA leaves before the other (cluster barrier); a CTA whose wait
 //     gave up pauses first, so that copies in flight land.
 // Key tiles are loaded without an L2 eviction hint: the pairs of different
 // query groups do not keep a fixed order over the same keys, so marking the
 // last group's loads evict-first let lines leave L2 before the other group
 // read them.
-constexpr int kPairStageBytes = 2 * kABytes;  // 128 x 64 keys + 128 x 64 queries
+constexpr int kPairStageBytes = 3 * kABytes;  // 2 x (128 x 64) keys + 128 x 64 queries
+constexpr int kPairUnitKeys = 4 * kTileM;     // keys per pair and step: two 256-key tiles
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
     tc_wide_pair_kernel(const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmQ, const WideArgs a)
 {
     constexpr int NM = 256;
     constexpr uint32_t kCols = 512;
-    constexpr int kPairKeys = 2 * kTileM;
 
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -762,23 +766,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
     const int q0 = group * NM;
     const int nqv = min(NM, a.B - q0);
 
-    const int64_t tiles = (a.N + kPairKeys - 1) / kPairKeys;
-    const int64_t t0 = tiles * part / a.parts, t1 = tiles * (part + 1) / a.parts;
-    const int64_t lo = t0 * kPairKeys;
-    const int64_t hi = min(a.N, t1 * kPairKeys);
-    const int ntiles = (int)(t1 - t0);
+    const int64_t units = (a.N + kPairUnitKeys - 1) / kPairUnitKeys;
+    const int64_t t0 = units * part / a.parts, t1 = units * (part + 1) / a.parts;
+    const int64_t lo = t0 * kPairUnitKeys;
+    const int64_t hi = min(a.N, t1 * kPairUnitKeys);
+    const int nunits = (int)(t1 - t0);
     const int kc = a.kchunks;
-    const int nsteps = ntiles * kc;
+    const int nsteps = nunits * kc;
 
     if (tid == 0) {
         for (int s = 0; s < a.stages; ++s) {
             mbar_init(&sh.full[s], 1);
             mbar_init(&sh.empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(&sh.acc_full[b], 1);
-            mbar_init(&sh.acc_empty[b], 2 * kEpiThreads);  // both CTAs' epilogue threads
-        }
+        mbar_init(&sh.acc_full[0], 1);
+        mbar_init(&sh.acc_empty[0], 2 * kWide2Epi);  // both CTAs' epilogue threads
         mbar_init(&sh.drain, 1);
         sh.abort = 0;
         sh.issued = 0;
@@ -807,9 +809,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
                 unsigned char* st = stages + (size_t)slot * kPairStageBytes;
                 const uint32_t full0 = full_base + (uint32_t)(slot * sizeof(uint64_t));
                 if (rank == 0) mbar_arrive_expect_tx(&sh.full[slot], 2 * kPairStageBytes);
-                const int32_t y = (int32_t)(lo + (int64_t)t * kPairKeys + kTileM * (int)rank);
+                // tile h of the unit is keys [base + 256 h, base + 256 h + 256);
+                // this CTA holds rows 128 rank .. 128 rank + 127 of each
+                const int32_t y = (int32_t)(lo + (int64_t)t * kPairUnitKeys + kTileM * (int)rank);
                 tma_load_2d_pair(st, &tmK, c * kChunkK, y, full0);
-                tma_load_2d_pair(st + kABytes, &tmQ, c * kChunkK, q0 + kTileM * (int)rank, full0);
+                tma_load_2d_pair(st + kABytes, &tmK, c * kChunkK, y + 2 * kTileM, full0);
+                tma_load_2d_pair(st + 2 * kABytes, &tmQ, c * kChunkK, q0 + kTileM * (int)rank,
+                                 full0);
                 *reinterpret_cast<volatile int*>(&sh.issued) = s + 1;
                 if (++slot == a.stages) {
                     slot = 0;
@@ -823,29 +829,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
             constexpr uint32_t idesc = mma_idesc_bf16(2 * kTileM, NM);
             int slot = 0;
             uint32_t phase = 0;
-            for (int j = 0; j < ntiles; ++j) {
-                const int buf = j & 1;
-                if (j >= 2)
-                    wait_or_abort_w(&sh.acc_empty[buf], (uint32_t)((j >> 1) - 1) & 1u, &sh.abort,
-                                    a.status);
+            for (int j = 0; j < nunits; ++j) {
+                if (j >= 1)
+                    wait_or_abort_w(&sh.acc_empty[0], (uint32_t)(j - 1) & 1u, &sh.abort, a.status);
                 tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)(buf * NM);
                 for (int c = 0; c < kc; ++c) {
                     wait_or_abort_w(&sh.full[slot], phase, &sh.abort, a.status);
                     tc_fence_after();
                     const unsigned char* st = stages + (size_t)slot * kPairStageBytes;
-                    const uint64_t ad = smem_desc_sw128(st);
-                    const uint64_t bd = smem_desc_sw128(st + kABytes);
+                    const uint64_t ad0 = smem_desc_sw128(st);
+                    const uint64_t ad1 = smem_desc_sw128(st + kABytes);
+                    const uint64_t bd = smem_desc_sw128(st + 2 * kABytes);
 #pragma unroll
-                    for (int k = 0; k < kChunkK / 16; ++k)
-                        mma_bf16_pair(d_tmem, ad + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
+                    for (int k = 0; k < kChunkK / 16; ++k) {
+                        mma_bf16_pair(tmem, ad0 + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
+                        mma_bf16_pair(tmem + (uint32_t)NM, ad1 + 2u * k, bd + 2u * k, idesc,
+                                      (c | k) != 0);
+                    }
                     mma_commit_pair_both(&sh.empty[slot]);
                     if (++slot == a.stages) {
                         slot = 0;
                         phase ^= 1u;
                     }
                 }
-                mma_commit_pair_both(&sh.acc_full[buf]);
+                mma_commit_pair_both(&sh.acc_full[0]);
             }
             // every MMA above has completed once this arrives
             mma_commit_pair_local(&sh.drain);
@@ -854,9 +861,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue (both CTAs)
-        const int e = tid - 64;
+        const int e = tid - 64;  // 0 .. 511
+        const int ew = warp - 2;  // 0 .. 15
         const int quarter = warp & 3;
-        for (int j = e; j < NM; j += kEpiThreads) {
+        const int h = (ew >> 2) & 1;              // 256-key tile of the unit this warp drains
+        const int c_base = (ew >> 3) * (NM / 2);  // first of the NM / 2 columns it drains
+        for (int j = e; j < NM; j += kWide2Epi) {
             // padding columns: -1 (never admitted); no sample threshold: every key
             uint32_t thr = 0xFFFFFFFFu;
             if (j < nqv) {
@@ -872,29 +882,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kTcThreads, 1)
                 a.cnt[q0 + j] = (int32_t)a.N;
             sh.qn[j] = j < nqv ? a.qn[q0 + j] : 0.f;
         }
-        named_barrier(2, kEpiThreads);
-        int2* resv = sh.resv + (warp - 2) * NM;
-        uint32_t* stage = &sh.stage[warp - 2][0][0];
-        wide_reserve(resv, 0, NM, nqv, lane, a, q0);
+        named_barrier(2, kWide2Epi);
+        // this warp's reservation entries, indexed by the absolute column
+        int2* resv = sh.resv + ew * (NM / 2) - c_base;
+        uint32_t* stage = &sh.stage[ew][0][0];
+        wide_reserve(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
 
         const int64_t ks = a.key_stride;
-        const int row_off = kTileM * (int)rank + 32 * quarter + lane;  // row within a 256-key tile
-        float kn_next = (ntiles > 0 && lo + row_off < hi) ? __ldg(a.knorm + (lo + row_off) * ks) : 0.f;
-        for (int j = 0; j < ntiles; ++j) {
-            const int buf = j & 1;
-            const int64_t row = lo + (int64_t)j * kPairKeys + row_off;
-            const float kn = kn_next;
-            kn_next = (row + kPairKeys < hi) ? __ldg(a.knorm + (row + kPairKeys) * ks) : 0.f;
+        const uint32_t tbase =
+            tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM + c_base);
+        const uint32_t release = mapa_shared(&sh.acc_empty[0], 0);
+        const int row_off = 2 * kTileM * h + kTileM * (int)rank + 32 * quarter + lane;
+        for (int j = 0; j < nunits; ++j) {
+            const int64_t row = lo + (int64_t)j * kPairUnitKeys + row_off;
+            const float kn = row < hi ? __ldg(a.knorm + row * ks) : 0.f;
             const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
             const int64_t pos = row < hi ? row : -1;
-            wait_or_abort_w(&sh.acc_full[buf], (uint32_t)(j >> 1) & 1u, &sh.abort, a.status);
+            wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
             tc_fence_after();
-            const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * NM);
-            wide_drain_row<NM, NM, true, true>(tbase, 0, nullptr, nqv, kn, valid,
-                                               (uint32_t)(row * ks), pos, lane, sh, resv, stage, a,
-                                               q0, mapa_shared(&sh.acc_empty[buf], 0));
+            wide_drain_row<NM, NM / 2, false, true>(tbase, c_base, nullptr, nqv, kn, valid,
+                                                    (uint32_t)(row * ks), pos, lane, sh, resv,
+                                                    stage, a, q0, release);
         }
-        wide_release(resv, 0, NM, nqv, lane, a, q0);
+        wide_release(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
     }
 
     tc_fence_before();
@@ -1214,11 +1224,11 @@ bool wide_plan_nm(size_t smem_limit, bool pairs, WidePlan* p)
     const size_t fixed = wide_fixed<NM>();
     p->pair = false;
     if (NM == 256 && pairs && fixed + 4 * (size_t)kPairStageBytes <= smem_limit) {
-        // CTA pairs: 32 KiB stages per CTA, double-buffered accumulators
+        // CTA pairs: 48 KiB stages per CTA (two 256-key tiles over the pair)
         int stages = (int)((smem_limit - fixed) / kPairStageBytes);
         stages = stages > kMaxStagesW ? kMaxStagesW : stages;
         p->nm = NM;
-        p->mb = 2;
+        p->mb = 4;
         p->pair = true;
         p->stages = stages;
         p->smem = fixed + (size_t)stages * kPairStageBytes;
@@ -1256,7 +1266,8 @@ cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUte
         cudaError_t e =
             raise_smem_limit(reinterpret_cast<const void*>(tc_wide_pair_kernel), (int)p.smem);
         if (e != cudaSuccess) return e;
-        tc_wide_pair_kernel<<<2 * p.groups * p.parts, kTcThreads, p.smem, stream>>>(tmK, tmQ, a);
+        tc_wide_pair_kernel<<<2 * p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ,
+                                                                                        a);
         return cudaGetLastError();
     }
     if (NM == 256 && p.mb == 2) {
@@ -1298,7 +1309,7 @@ int wide_pair_clusters(size_t smem_limit)
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2, 1, 1);
-    cfg.blockDim = dim3(kTcThreads, 1, 1);
+    cfg.blockDim = dim3(kWide2Threads, 1, 1);
     cfg.dynamicSmemBytes = p.smem;
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(tc_wide_pair_kernel),

@@ -94,19 +94,25 @@ def load_library(path: str | None = None):
     return lib
 
 
+def _pair_mode(on: bool | None) -> int:
+    """nest_datastore_use_cta_pairs mode: 1 (pairs), 0 (single CTAs), -1 (automatic)."""
+    return -1 if on is None else int(bool(on))
+
+
 def plan_offline(N: int, d: int, dtype: str, B: int, r: int, ragged: bool = False,
                  num_sms: int = 152, smem_per_block: int = 232448,
-                 cta_pairs: bool = False) -> dict:
+                 cta_pairs: bool | None = None) -> dict:
     """The plan a search of this shape would run (nest_plan_offline): host
     only, no GPU.  The defaults are a GB300's 152 SMs and 227 KiB of opt-in
-    shared memory per block.  ``dtype`` is "f32" or "bf16"."""
+    shared memory per block.  ``dtype`` is "f32" or "bf16".  ``cta_pairs``
+    as in Datastore.use_cta_pairs (None: the handle's automatic default)."""
     lib = load_library()
     p = Plan()
     code = BF16 if dtype == "bf16" else F32 if dtype == "f32" else -1
     if code < 0:
         raise ValueError("dtype must be 'f32' or 'bf16'")
     _check(lib.nest_plan_offline(int(N), int(d), code, int(B), int(r), int(bool(ragged)),
-                                 int(num_sms), int(smem_per_block), int(bool(cta_pairs)),
+                                 int(num_sms), int(smem_per_block), _pair_mode(cta_pairs),
                                  ctypes.byref(p)), "nest_plan_offline")
     out = {name: getattr(p, name) for name, _ in Plan._fields_}
     out["kernel"] = Datastore.SEARCH_PATHS[p.path]
@@ -192,10 +198,11 @@ class Datastore:
         _check(self._lib.nest_datastore_reserve(self._h, max_B, max_r, int(ragged)),
                "nest_datastore_reserve")
 
-    def use_cta_pairs(self, on: bool) -> None:
-        """Groups of 256 queries on CTA pairs (opt-in) or on single CTAs with
-        two key tiles per stage (default)."""
-        _check(self._lib.nest_datastore_use_cta_pairs(self._h, int(bool(on))),
+    def use_cta_pairs(self, on: bool | None) -> None:
+        """Groups of 256 queries on CTA pairs (True), on single CTAs with two
+        key tiles per stage (False), or automatically (None, the default):
+        pairs when the batch is one group."""
+        _check(self._lib.nest_datastore_use_cta_pairs(self._h, _pair_mode(on)),
                "nest_datastore_use_cta_pairs")
 
     # ------------------------------------------------------------ search / mix / step

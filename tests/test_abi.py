@@ -133,6 +133,9 @@ def test_nest_step_calls_validation(lib):
     assert lib.nest_verify_spans(ds, P(FAKE + 2), a, 1, a, 1, 0.5, a, a, a, None) == 3
     # handle-level calls
     assert lib.nest_datastore_use_cta_pairs(None, 1) == 1
+    # modes are 1, 0 and -1 (checked before the handle is read)
+    assert lib.nest_datastore_use_cta_pairs(ds, 2) == 1
+    assert lib.nest_datastore_use_cta_pairs(ds, -2) == 1
     assert lib.nest_selftest_bounded_wait(None, None, None) == 1
     assert lib.nest_datastore_reserve(None, 1, 1, 0) == 1
     assert lib.nest_search_path(None, 1, 1, 0) == -1

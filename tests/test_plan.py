@@ -61,6 +61,24 @@ def test_large_batch_plan(nest):
     assert (q["groups"], q["parts"]) == (2, SMS // 4)  # 2 groups x 38 pairs = 152 SMs
 
 
+def test_hidden8192_plan_runs_one_group_on_cta_pairs(nest):
+    """B=256 at d=8192 over 8M keys is one group of 256 queries: by default
+    it runs on 76 CTA pairs (two 256-key tiles per 48 KiB stage, four
+    stages); forced off, on 152 single CTAs with three 64 KiB stages."""
+    p = nest.plan_offline(1 << 23, 8192, "bf16", 256, 1024, num_sms=SMS, smem_per_block=SMEM)
+    assert p["kernel"] == "tc_wide_pair_kernel"
+    assert (p["groups"], p["parts"], p["stages"]) == (1, SMS // 2, 4)
+    q = nest.plan_offline(1 << 23, 8192, "bf16", 256, 1024, num_sms=SMS, smem_per_block=SMEM,
+                          cta_pairs=False)
+    assert q["kernel"] == "tc_wide2_kernel"
+    assert (q["groups"], q["parts"], q["stages"]) == (1, SMS, 3)
+    # batches of 129 to 256 queries are one group; more are several
+    for B, kernel in ((129, "tc_wide_pair_kernel"), (128, "tc_wide_kernel"),
+                      (257, "tc_wide2_kernel")):
+        assert nest.plan_offline(1 << 23, 8192, "bf16", B, 1024, num_sms=SMS,
+                                 smem_per_block=SMEM)["kernel"] == kernel, B
+
+
 def test_ragged_and_fp32_plans(nest):
     p = nest.plan_offline(32 * 10240, 4096, "bf16", 32, 64, ragged=True, num_sms=SMS,
                           smem_per_block=SMEM)
@@ -104,7 +122,8 @@ def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
             assert p["scratch_bytes"] >= groups * p["parts"] * qpg * r * 8, tag
         else:
             assert not c["ragged"] and c["dtype"] == "bf16", tag
-            assert (p["path"] == 4) == (pairs_of(c) and qpg == 256), tag
+            # pairs when forced, or automatically for a single group of 256
+            assert (p["path"] == 4) == (qpg == 256 and (pairs_of(c) or groups == 1)), tag
             if p["single_pass"]:
                 assert p["sample_stride"] == 1 and p["list_capacity"] == N, tag
             else:
