@@ -107,21 +107,27 @@ NEST_API nest_status_t nest_datastore_reserve(nest_datastore_t* ds, int32_t max_
                                      int32_t ragged);
 
 /*
- * How searches with groups of 256 queries are laid out on the SMs (search
+ * How searches of more than 128 queries are laid out on the SMs (search
  * paths 3 and 4 of nest_search_path).  Both return the same neighbours.
  *
  *   mode  1  always on CTA pairs (path 4): each 256-key tile is split over
- *            the two SMs of a pair and each CTA stages only half of the
- *            group's queries, so a pipeline stage carries the MMA work of a
+ *            the two SMs of a pair and each CTA stages only half of each
+ *            256-query block, so a pipeline stage carries the MMA work of a
  *            path-3 stage in three quarters of the shared memory (four
- *            stages instead of three).
- *   mode  0  never: single CTAs with two 128-key tiles per stage (path 3).
+ *            stages instead of three).  Batches of 257 to 512 queries run as
+ *            one group of 512 (one 256-key tile against both halves per
+ *            stage); other batches as groups of 256 (two 256-key tiles per
+ *            stage).
+ *   mode  0  never: single CTAs with two 128-key tiles per stage and groups
+ *            of 256 queries (path 3).
  *   mode -1  automatic, the default: pairs when the batch is one group
- *            (129 to 256 queries), single CTAs for more groups.  With one
- *            group the pairs' main pass is about 4 % faster (d = 8192,
- *            8M keys, B = 256 on a GB300); with several groups their pairs
- *            drift apart over the same keys and read them from DRAM again,
- *            which made them about 5 % slower (4M keys, B = 512).
+ *            (129 to 512 queries), single CTAs for more.  On a GB300, pairs
+ *            made the main pass about 5 % faster at d = 8192, 8M keys,
+ *            B = 256, and about 3 % faster at d = 4096, 4M keys, B = 512
+ *            (every key read from DRAM once instead of once per group of
+ *            256).  Two or more pair groups drift apart over the same keys
+ *            and read them from DRAM again, so larger batches stay on single
+ *            CTAs, whose four or more groups share the keys in L2.
  *
  * Pairs need two CTAs of about 220 KiB of shared memory each on the two SMs
  * of one TPC at the same time; mode 1 where the device cannot place them
@@ -385,9 +391,9 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
  *      thresholds (bf16 keys, more queries than one CTA keeps lists for)
  *   3  the same with two 128-key tiles per pipeline stage (groups of 256
  *      queries, when three 64 KiB stages fit in shared memory)
- *   4  the same on CTA pairs (groups of 256 queries, 256-key tiles split
- *      over two SMs, two such tiles per stage): by default when the batch
- *      is one group; see nest_datastore_use_cta_pairs
+ *   4  the same on CTA pairs (groups of 256 or 512 queries, 256-key tiles
+ *      split over two SMs): by default for 129 to 512 queries; see
+ *      nest_datastore_use_cta_pairs
  * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
  */
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,
@@ -431,8 +437,9 @@ NEST_API int64_t nest_launch_count(const nest_datastore_t* ds);
 NEST_API const char* nest_status_string(nest_status_t status);
 
 /* ABI version: major * 10000 + minor * 100 + patch (0.2.0: CTA pairs and
- * the bounded-wait self-test added to 0.1.0; 0.3.0: CTA pairs with two
- * 256-key tiles per stage, chosen automatically for one query group). */
+ * the bounded-wait self-test added to 0.1.0; 0.3.0: CTA pairs with 48 KiB
+ * stages and groups of up to 512 queries, chosen automatically for one
+ * query group). */
 NEST_API int32_t nest_version(void);
 
 #ifdef __cplusplus

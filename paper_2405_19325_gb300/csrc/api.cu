@@ -188,16 +188,23 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
     sp->total_words = sp->off_fin + fin_words;
     sp->wide = false;
     // More queries than one CTA can keep lists for: stream the keys once per
-    // group of up to 256 queries against sampled admission thresholds.
+    // group of up to 256 queries (512 on CTA pairs) against sampled
+    // admission thresholds.
     if (sp->tc && !ragged && sp->groups > 1) {
-        const int nm = B >= 256 ? 256 : std::max(16, ceil_pow2(B));
-        WidePlan wp{};
         // CTA pairs: when asked for, or (automatic) when the batch is one
-        // group, whose key ranges no other group's CTAs stream beside them
-        const bool one_group = B <= nm;
+        // group of up to 512, whose key ranges no other group's CTAs stream
+        // beside them
         const bool pairs =
-            ds->pairs_ok && (ds->pairs_mode == 1 || (ds->pairs_mode < 0 && one_group));
-        if (wide_plan_smem(nm, ds->smem_optin, pairs, &wp)) {
+            ds->pairs_ok && (ds->pairs_mode == 1 || (ds->pairs_mode < 0 && B <= 512));
+        int nm = B >= 256 ? 256 : std::max(16, ceil_pow2(B));
+        if (pairs && B > 256 && B <= 512) nm = 512;  // one pair group of 512
+        WidePlan wp{};
+        bool planned = wide_plan_smem(nm, ds->smem_optin, pairs, &wp);
+        if (!planned && nm == 512) {
+            nm = 256;
+            planned = wide_plan_smem(nm, ds->smem_optin, false, &wp);
+        }
+        if (planned) {
             wp.groups = (B + nm - 1) / nm;
             // A sample of every stride-th key, about max(65,536, 64 r) keys.
             const int64_t target = std::max<int64_t>(65536, 64 * (int64_t)r);
@@ -241,15 +248,16 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
             sp->resv = (int32_t)std::min<int64_t>(2 * per_warp + 16, 1024);
             const int64_t unwritten = (int64_t)sp->wpm.parts * epi_warps * sp->resv;
             sp->cap_m = std::min<int64_t>(ds->N, std::max<int64_t>(8LL * r, 8 * expect)) + unwritten;
-            // recovery of overflowed main-pass lists: the same groups, one
-            // 128-key tile per stage
-            if (!wide_recover_plan(nm, ds->smem_optin, &sp->wpr)) return NEST_ERR_UNSUPPORTED;
-            sp->wpr.groups = wp.groups;
-            sp->wpr.parts = choose_parts(wp.groups, ds->N, ds->num_sms, false);
-            // 2 * B int32 counters, then kRecoverRounds * groups int32 flags
-            // (zeroed by one memset per search)
+            // recovery of overflowed main-pass lists: groups of up to 256
+            // queries (a group of 512 as two), one 128-key tile per stage
+            const int nr = std::min(nm, 256);
+            if (!wide_recover_plan(nr, ds->smem_optin, &sp->wpr)) return NEST_ERR_UNSUPPORTED;
+            sp->wpr.groups = (B + nr - 1) / nr;
+            sp->wpr.parts = choose_parts(sp->wpr.groups, ds->N, ds->num_sms, false);
+            // 2 * B int32 counters, then kRecoverRounds * recovery groups
+            // int32 flags (zeroed by one memset per search)
             sp->off_cnt = 0;
-            sp->cnt_ints = 2 * (size_t)B + (size_t)kRecoverRounds * wp.groups;
+            sp->cnt_ints = 2 * (size_t)B + (size_t)kRecoverRounds * sp->wpr.groups;
             sp->off_qn = (sp->cnt_ints + 1) / 2;
             sp->off_lim = sp->off_qn + ((size_t)B + 1) / 2;  // after B floats ||q||^2
             sp->off_cand_s = sp->off_lim + (size_t)B;       // after B word limits
@@ -472,8 +480,8 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
     cudaError_t e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * sp.cnt_ints, stream);
     if (e != cudaSuccess) return from_cuda(e);
     CUtensorMap qmap;
-    // a CTA of a pair stages half of the group's queries
-    if (!encode_bf16_rows(&qmap, q, B, ds->d, sp.wpm.pair ? sp.wpm.nm / 2 : sp.wpm.nm, false))
+    // a CTA of a pair stages 128 queries of each 256 of the group
+    if (!encode_bf16_rows(&qmap, q, B, ds->d, sp.wpm.pair ? 128 : sp.wpm.nm, false))
         return NEST_ERR_CUDA;
 
     WideArgs wa{};
@@ -576,14 +584,15 @@ nest_status_t launch_wide(nest_datastore* ds, const SearchPlan& sp, const void* 
         gp.r = r;
         gp.B = B;
         gp.lim_out = lim;
-        gp.group_flag = flags + (size_t)round * sp.wpm.groups;
-        gp.group_size = sp.wpm.nm;
+        gp.group_flag = flags + (size_t)round * sp.wpr.groups;
+        gp.group_size = sp.wpr.nm;
         gp.s_sample = s_s;
         gp.check_underflow = round == 0 ? 1 : 0;
         e = launch_gselect(gp, stream);
         if (e != cudaSuccess) return from_cuda(e);
         WideArgs wr = wa;
         wr.resv = 0;
+        wr.groups = sp.wpr.groups;
         wr.parts = sp.wpr.parts;
         wr.stages = sp.wpr.stages;
         wr.word_lim = lim;

@@ -14,8 +14,8 @@
 //      K = 16): tc_wide_kernel keeps one key tile per stage and two TMEM
 //      accumulators of N columns.  Groups of 256 run on tc_wide2_kernel
 //      (two key tiles per stage, one accumulator each) or on CTA pairs
-//      (tc_wide_pair_kernel: M = 256 keys over the pair, two such tiles per
-//      stage; the default when the batch is one group).  The epilogue warps form
+//      (tc_wide_pair_kernel: M = 256 keys over the pair; the default when
+//      the batch is one group of up to 512 queries).  The epilogue warps form
 //      ||q||^2 + ||k||^2 - 2 q.k, admit the keys under each query's threshold
 //      and append them to that query's global list through per-warp slot
 //      reservations.
@@ -50,8 +50,9 @@ struct WideShared {
     // Slots [x, y) of query column c's global list reserved by an epilogue
     // warp and not yet written (used when WideArgs::resv > 0); x passes y
     // once the block is used up.  Each warp has one entry per column it
-    // drains (NM / 2 or NM columns).
-    int2 resv[8 * NM];
+    // drains (NM / 2 or NM columns; 128 in each of a CTA pair's sixteen
+    // epilogue warps for groups of 512).
+    int2 resv[NM <= 256 ? 8 * NM : 16 * 128];
     // Distance bits of the keys a lane admitted in one 32-column block, in
     // column order: [warp][k][lane].
     uint32_t stage[kMaxEpiWarps][kStageK][32];
@@ -719,17 +720,22 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
     }
 }
 
-// Groups of 256 queries on CTA pairs (a cluster of two CTAs on one TPC):
-// tcgen05.mma.cta_group::2 with M = 256 keys (128 in each CTA's shared
+// Groups of 256 or 512 queries on CTA pairs (a cluster of two CTAs on one
+// TPC): tcgen05.mma.cta_group::2 with M = 256 keys (128 in each CTA's shared
 // memory and TMEM lanes), N = 256 queries (each CTA stages 128 of them; the
-// MMA reads both halves) and K = 16, two such 256-key tiles per stage.  Per
-// CTA a stage is 32 KiB of keys and 16 KiB of queries, where the two-tile
-// kernel above stages 32 KiB of keys and the whole 32 KiB query chunk for
-// the same MMA work per SM: the pair reads half as many query bytes from L2
-// and four 48 KiB stages fit where three 64 KiB stages did, so the ring
-// covers a third more latency.  Each CTA's two 256-column accumulators fill
-// its TMEM, so, as in the two-tile kernel, a tile pair's epilogue runs
-// between its last MMA and the next pair's first.
+// MMA reads both halves) and K = 16.  Each CTA's TMEM holds two 256-column
+// accumulators, filled in one of two ways:
+//   MT = 2  groups of 256 queries, two 256-key tiles per stage;
+//   MT = 1  groups of 512 queries, one 256-key tile per stage against both
+//           256-query halves, so a batch of up to 512 queries reads every key
+//           from DRAM once instead of once per group of 256.
+// Either way a stage is 48 KiB per CTA (three 16 KiB blocks of 128 x 64 bf16:
+// key rows, then query rows), where the single-CTA two-tile kernel above
+// stages 64 KiB for the same MMA work per SM: the pair reads fewer query
+// bytes from L2 per key byte, and four stages fit where three did, so the
+// ring covers a third more latency.  The accumulators fill TMEM, so, as in
+// the two-tile kernel, a step's epilogue runs between its last MMA and the
+// next step's first.
 //   * both CTAs' TMA loads complete on the even CTA's full barrier, which the
 //     even CTA arms with the pair's bytes; the even CTA's MMA thread issues
 //     for the pair and its commits arrive on both CTAs' empty and acc_full
@@ -742,14 +748,17 @@ __global__ void __launch_bounds__(kWide2Threads, 1)
 // query groups do not keep a fixed order over the same keys, so marking the
 // last group's loads evict-first let lines leave L2 before the other group
 // read them.
-constexpr int kPairStageBytes = 3 * kABytes;  // 2 x (128 x 64) keys + 128 x 64 queries
-constexpr int kPairUnitKeys = 4 * kTileM;     // keys per pair and step: two 256-key tiles
+constexpr int kPairStageBytes = 3 * kABytes;  // key and query blocks of 128 x 64 per CTA
 
+template <int MT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
     tc_wide_pair_kernel(const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmQ, const WideArgs a)
 {
-    constexpr int NM = 256;
+    static_assert(MT == 1 || MT == 2, "one or two 256-key tiles per stage");
+    constexpr int NG = 2 / MT;               // 256-query halves of the group
+    constexpr int NM = 256 * NG;             // queries of the group
+    constexpr int kUnitKeys = 2 * kTileM * MT;  // keys per pair and step
     constexpr uint32_t kCols = 512;
 
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -766,10 +775,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
     const int q0 = group * NM;
     const int nqv = min(NM, a.B - q0);
 
-    const int64_t units = (a.N + kPairUnitKeys - 1) / kPairUnitKeys;
+    const int64_t units = (a.N + kUnitKeys - 1) / kUnitKeys;
     const int64_t t0 = units * part / a.parts, t1 = units * (part + 1) / a.parts;
-    const int64_t lo = t0 * kPairUnitKeys;
-    const int64_t hi = min(a.N, t1 * kPairUnitKeys);
+    const int64_t lo = t0 * kUnitKeys;
+    const int64_t hi = min(a.N, t1 * kUnitKeys);
     const int nunits = (int)(t1 - t0);
     const int kc = a.kchunks;
     const int nsteps = nunits * kc;
@@ -809,13 +818,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
                 unsigned char* st = stages + (size_t)slot * kPairStageBytes;
                 const uint32_t full0 = full_base + (uint32_t)(slot * sizeof(uint64_t));
                 if (rank == 0) mbar_arrive_expect_tx(&sh.full[slot], 2 * kPairStageBytes);
-                // tile h of the unit is keys [base + 256 h, base + 256 h + 256);
-                // this CTA holds rows 128 rank .. 128 rank + 127 of each
-                const int32_t y = (int32_t)(lo + (int64_t)t * kPairUnitKeys + kTileM * (int)rank);
-                tma_load_2d_pair(st, &tmK, c * kChunkK, y, full0);
-                tma_load_2d_pair(st + kABytes, &tmK, c * kChunkK, y + 2 * kTileM, full0);
-                tma_load_2d_pair(st + 2 * kABytes, &tmQ, c * kChunkK, q0 + kTileM * (int)rank,
-                                 full0);
+                // key tile tt of the step is keys [base + 256 tt, base + 256 tt + 256)
+                // and query half g is queries [q0 + 256 g, q0 + 256 g + 256); this
+                // CTA holds rows 128 rank .. 128 rank + 127 of each
+                const int32_t y = (int32_t)(lo + (int64_t)t * kUnitKeys + kTileM * (int)rank);
+#pragma unroll
+                for (int tt = 0; tt < MT; ++tt)
+                    tma_load_2d_pair(st + tt * kABytes, &tmK, c * kChunkK, y + 2 * kTileM * tt,
+                                     full0);
+#pragma unroll
+                for (int g = 0; g < NG; ++g)
+                    tma_load_2d_pair(st + (MT + g) * kABytes, &tmQ, c * kChunkK,
+                                     q0 + 2 * kTileM * g + kTileM * (int)rank, full0);
                 *reinterpret_cast<volatile int*>(&sh.issued) = s + 1;
                 if (++slot == a.stages) {
                     slot = 0;
@@ -826,7 +840,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer (even CTA)
         if (rank == 0 && lane == 0 && nsteps > 0) {
-            constexpr uint32_t idesc = mma_idesc_bf16(2 * kTileM, NM);
+            constexpr uint32_t idesc = mma_idesc_bf16(2 * kTileM, 256);
             int slot = 0;
             uint32_t phase = 0;
             for (int j = 0; j < nunits; ++j) {
@@ -837,14 +851,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
                     wait_or_abort_w(&sh.full[slot], phase, &sh.abort, a.status);
                     tc_fence_after();
                     const unsigned char* st = stages + (size_t)slot * kPairStageBytes;
-                    const uint64_t ad0 = smem_desc_sw128(st);
-                    const uint64_t ad1 = smem_desc_sw128(st + kABytes);
-                    const uint64_t bd = smem_desc_sw128(st + 2 * kABytes);
 #pragma unroll
                     for (int k = 0; k < kChunkK / 16; ++k) {
-                        mma_bf16_pair(tmem, ad0 + 2u * k, bd + 2u * k, idesc, (c | k) != 0);
-                        mma_bf16_pair(tmem + (uint32_t)NM, ad1 + 2u * k, bd + 2u * k, idesc,
-                                      (c | k) != 0);
+                        // accumulator tt * NG + g: key tile tt against query half g
+#pragma unroll
+                        for (int tt = 0; tt < MT; ++tt)
+#pragma unroll
+                            for (int g = 0; g < NG; ++g)
+                                mma_bf16_pair(tmem + (uint32_t)(256 * (tt * NG + g)),
+                                              smem_desc_sw128(st + tt * kABytes) + 2u * k,
+                                              smem_desc_sw128(st + (MT + g) * kABytes) + 2u * k,
+                                              idesc, (c | k) != 0);
                     }
                     mma_commit_pair_both(&sh.empty[slot]);
                     if (++slot == a.stages) {
@@ -864,8 +881,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
         const int e = tid - 64;  // 0 .. 511
         const int ew = warp - 2;  // 0 .. 15
         const int quarter = warp & 3;
-        const int h = (ew >> 2) & 1;              // 256-key tile of the unit this warp drains
-        const int c_base = (ew >> 3) * (NM / 2);  // first of the NM / 2 columns it drains
+        const int acc = (ew >> 2) & 1;            // accumulator this warp drains
+        const int tt = MT == 2 ? acc : 0;         // its key tile
+        const int g = MT == 2 ? 0 : acc;          // its query half
+        const int c_base = (ew >> 3) * 128;       // first of its 128 columns in the accumulator
+        const int col0 = 256 * g + c_base;        // ... as a query of the group
         for (int j = e; j < NM; j += kWide2Epi) {
             // padding columns: -1 (never admitted); no sample threshold: every key
             uint32_t thr = 0xFFFFFFFFu;
@@ -883,28 +903,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kWide2Threads, 1)
             sh.qn[j] = j < nqv ? a.qn[q0 + j] : 0.f;
         }
         named_barrier(2, kWide2Epi);
-        // this warp's reservation entries, indexed by the absolute column
-        int2* resv = sh.resv + ew * (NM / 2) - c_base;
+        // this warp's reservation entries, indexed by the query of the group
+        int2* resv = sh.resv + ew * 128 - col0;
         uint32_t* stage = &sh.stage[ew][0][0];
-        wide_reserve(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
+        wide_reserve(resv, col0, col0 + 128, nqv, lane, a, q0);
 
         const int64_t ks = a.key_stride;
         const uint32_t tbase =
-            tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(h * NM + c_base);
+            tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(256 * acc + c_base);
         const uint32_t release = mapa_shared(&sh.acc_empty[0], 0);
-        const int row_off = 2 * kTileM * h + kTileM * (int)rank + 32 * quarter + lane;
+        const int row_off = 2 * kTileM * tt + kTileM * (int)rank + 32 * quarter + lane;
         for (int j = 0; j < nunits; ++j) {
-            const int64_t row = lo + (int64_t)j * kPairUnitKeys + row_off;
+            const int64_t row = lo + (int64_t)j * kUnitKeys + row_off;
             const float kn = row < hi ? __ldg(a.knorm + row * ks) : 0.f;
             const bool valid = row < hi && !key_masked(a.key_mask, row * ks);
             const int64_t pos = row < hi ? row : -1;
             wait_or_abort_w(&sh.acc_full[0], (uint32_t)j & 1u, &sh.abort, a.status);
             tc_fence_after();
-            wide_drain_row<NM, NM / 2, false, true>(tbase, c_base, nullptr, nqv, kn, valid,
-                                                    (uint32_t)(row * ks), pos, lane, sh, resv,
-                                                    stage, a, q0, release);
+            wide_drain_row<NM, 128, false, true>(tbase, col0, nullptr, nqv, kn, valid,
+                                                 (uint32_t)(row * ks), pos, lane, sh, resv, stage,
+                                                 a, q0, release);
         }
-        wide_release(resv, c_base, c_base + NM / 2, nqv, lane, a, q0);
+        wide_release(resv, col0, col0 + 128, nqv, lane, a, q0);
     }
 
     tc_fence_before();
@@ -1223,17 +1243,19 @@ bool wide_plan_nm(size_t smem_limit, bool pairs, WidePlan* p)
 {
     const size_t fixed = wide_fixed<NM>();
     p->pair = false;
-    if (NM == 256 && pairs && fixed + 4 * (size_t)kPairStageBytes <= smem_limit) {
-        // CTA pairs: 48 KiB stages per CTA (two 256-key tiles over the pair)
+    if (NM >= 256 && pairs && fixed + 4 * (size_t)kPairStageBytes <= smem_limit) {
+        // CTA pairs: 48 KiB stages per CTA; groups of 256 take two 256-key
+        // tiles per step, groups of 512 one
         int stages = (int)((smem_limit - fixed) / kPairStageBytes);
         stages = stages > kMaxStagesW ? kMaxStagesW : stages;
         p->nm = NM;
-        p->mb = 4;
+        p->mb = NM == 256 ? 4 : 2;
         p->pair = true;
         p->stages = stages;
         p->smem = fixed + (size_t)stages * kPairStageBytes;
         return true;
     }
+    if (NM > 256) return false;  // groups of 512 run on pairs only
     if (NM == 256) {
         // two key tiles per stage when three 64 KiB stages fit
         const size_t st2 = (size_t)(2 * kABytes + NM * kChunkK * 2);
@@ -1262,26 +1284,31 @@ template <int NM>
 cudaError_t wide_launch_nm(const WidePlan& p, const CUtensorMap& tmK, const CUtensorMap& tmQ,
                            const WideArgs& a, cudaStream_t stream)
 {
-    if (NM == 256 && p.pair) {
-        cudaError_t e =
-            raise_smem_limit(reinterpret_cast<const void*>(tc_wide_pair_kernel), (int)p.smem);
-        if (e != cudaSuccess) return e;
-        tc_wide_pair_kernel<<<2 * p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ,
-                                                                                        a);
-        return cudaGetLastError();
+    if constexpr (NM >= 256) {
+        if (p.pair) {
+            auto kern = tc_wide_pair_kernel<NM == 256 ? 2 : 1>;
+            cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
+            if (e != cudaSuccess) return e;
+            kern<<<2 * p.groups * p.parts, kWide2Threads, p.smem, stream>>>(tmK, tmQ, a);
+            return cudaGetLastError();
+        }
     }
-    if (NM == 256 && p.mb == 2) {
-        cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_wide2_kernel), (int)p.smem);
+    if constexpr (NM > 256) {
+        return cudaErrorInvalidValue;  // groups of 512 run on pairs only
+    } else {
+        if (NM == 256 && p.mb == 2) {
+            cudaError_t e =
+                raise_smem_limit(reinterpret_cast<const void*>(tc_wide2_kernel), (int)p.smem);
+            if (e != cudaSuccess) return e;
+            return launch_pdl(tc_wide2_kernel, dim3(p.groups * p.parts), dim3(kWide2Threads),
+                              p.smem, stream, tmK, tmQ, a);
+        }
+        auto kern = tc_wide_kernel<NM>;
+        cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
         if (e != cudaSuccess) return e;
-        return launch_pdl(tc_wide2_kernel, dim3(p.groups * p.parts), dim3(kWide2Threads), p.smem,
-                          stream, tmK, tmQ, a);
+        return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kTcThreads), p.smem, stream, tmK,
+                          tmQ, a);
     }
-    auto kern = tc_wide_kernel<NM>;
-    cudaError_t e =
-        raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem);
-    if (e != cudaSuccess) return e;
-    return launch_pdl(kern, dim3(p.groups * p.parts), dim3(kTcThreads), p.smem, stream, tmK, tmQ,
-                      a);
 }
 
 }  // namespace
@@ -1294,16 +1321,22 @@ bool wide_plan_smem(int nm, size_t smem_limit, bool pairs, WidePlan* p)
     case 64: return wide_plan_nm<64>(smem_limit, pairs, p);
     case 128: return wide_plan_nm<128>(smem_limit, pairs, p);
     case 256: return wide_plan_nm<256>(smem_limit, pairs, p);
+    case 512: return wide_plan_nm<512>(smem_limit, pairs, p);
     default: return false;
     }
 }
 
-int wide_pair_clusters(size_t smem_limit)
+namespace {
+
+// Clusters of the pair kernel for groups of NM queries that the device can
+// hold at once (0: none, or the plan does not fit).
+template <int NM>
+int pair_clusters_nm(size_t smem_limit)
 {
     WidePlan p{};
-    if (!wide_plan_nm<256>(smem_limit, true, &p) || !p.pair) return 0;
-    if (raise_smem_limit(reinterpret_cast<const void*>(tc_wide_pair_kernel), (int)p.smem) !=
-        cudaSuccess) {
+    if (!wide_plan_nm<NM>(smem_limit, true, &p) || !p.pair) return 0;
+    auto kern = tc_wide_pair_kernel<NM == 256 ? 2 : 1>;
+    if (raise_smem_limit(reinterpret_cast<const void*>(kern), (int)p.smem) != cudaSuccess) {
         (void)cudaGetLastError();
         return 0;
     }
@@ -1312,12 +1345,21 @@ int wide_pair_clusters(size_t smem_limit)
     cfg.blockDim = dim3(kWide2Threads, 1, 1);
     cfg.dynamicSmemBytes = p.smem;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(tc_wide_pair_kernel),
-                                       &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) !=
+        cudaSuccess) {
         (void)cudaGetLastError();
         return 0;
     }
     return n;
+}
+
+}  // namespace
+
+int wide_pair_clusters(size_t smem_limit)
+{
+    const int a = pair_clusters_nm<256>(smem_limit);
+    const int b = pair_clusters_nm<512>(smem_limit);
+    return a < b ? a : b;
 }
 
 namespace {
@@ -1385,6 +1427,7 @@ cudaError_t launch_tc_wide(const WidePlan& p, const CUtensorMap& tmK, const CUte
     case 64: return wide_launch_nm<64>(p, tmK, tmQ, a, stream);
     case 128: return wide_launch_nm<128>(p, tmK, tmQ, a, stream);
     case 256: return wide_launch_nm<256>(p, tmK, tmQ, a, stream);
+    case 512: return wide_launch_nm<512>(p, tmK, tmQ, a, stream);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -199,9 +199,9 @@ class Datastore:
                "nest_datastore_reserve")
 
     def use_cta_pairs(self, on: bool | None) -> None:
-        """Groups of 256 queries on CTA pairs (True), on single CTAs with two
-        key tiles per stage (False), or automatically (None, the default):
-        pairs when the batch is one group."""
+        """Batches of more than 128 queries on CTA pairs (True), on single
+        CTAs with two key tiles per stage (False), or automatically (None,
+        the default): pairs when the batch is one group (up to 512)."""
         _check(self._lib.nest_datastore_use_cta_pairs(self._h, _pair_mode(on)),
                "nest_datastore_use_cta_pairs")
 

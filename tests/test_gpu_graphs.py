@@ -42,6 +42,7 @@ def _case(N, d, B, vocab, seed):
 @pytest.mark.parametrize("N,d,B,r,path", [
     (200000, 1024, 4, 256, "tc_scan_kernel"),      # decode-shaped: scan + merge + mix
     (100000, 256, 40, 128, "tc_wide_kernel"),      # large batch: sample, main pass, selections
+    (140000, 128, 300, 64, "tc_wide_pair_kernel"),  # one group of 512 on CTA pairs (clusters)
 ])
 def test_captured_step_replays_match_eager(nest, N, d, B, r, path):
     vocab = 1000

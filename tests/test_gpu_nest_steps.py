@@ -110,8 +110,8 @@ def test_verify_spans_matches_oracle(nest):
 def test_masked_search_skips_used_keys(nest, path, B, r, dtype, N):
     K, V, q, p_lm = _case(N, 256, B, 300, seed=42, dtype=dtype)
     ds = nest.Datastore(K, V, 300)
-    if path == "tc_wide_pair_kernel":
-        ds.use_cta_pairs(True)
+    if path in ("tc_wide_pair_kernel", "tc_wide2_kernel"):
+        ds.use_cta_pairs(path == "tc_wide_pair_kernel")
     assert ds.search_path(B, r) == path
     mask = ds.new_key_mask()
     g = torch.Generator().manual_seed(43)

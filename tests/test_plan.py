@@ -50,15 +50,20 @@ def test_large_batch_plan(nest):
     for the exact re-ranking).  The main pass admits keys up to the sample's
     32nd distance: about 32 x 64 = 2,048 survivors per query, and the lists
     hold 8x that."""
-    p = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM)
+    p = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
+                          cta_pairs=False)
     assert p["kernel"] == "tc_wide2_kernel"
     assert (p["queries_per_group"], p["groups"], p["parts"]) == (256, 2, SMS // 2)
     assert p["single_pass"] == 0 and p["sample_stride"] == (1 << 22) // 65536
     assert p["list_capacity"] >= 8 * 32 * 64  # 8x the expected survivors
-    q = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
-                          cta_pairs=True)
-    assert q["kernel"] == "tc_wide_pair_kernel"
-    assert (q["groups"], q["parts"]) == (2, SMS // 4)  # 2 groups x 38 pairs = 152 SMs
+    # by default (and when forced) the 512 queries are one group on 76 CTA pairs,
+    # each pair streaming its key range once for all of them
+    for mode in (None, True):
+        q = nest.plan_offline(1 << 22, 4096, "bf16", 512, 256, num_sms=SMS, smem_per_block=SMEM,
+                              cta_pairs=mode)
+        assert q["kernel"] == "tc_wide_pair_kernel"
+        assert (q["queries_per_group"], q["groups"], q["parts"], q["stages"]) == (512, 1, SMS // 2, 4)
+        assert q["sample_stride"] == p["sample_stride"]
 
 
 def test_hidden8192_plan_runs_one_group_on_cta_pairs(nest):
@@ -72,9 +77,10 @@ def test_hidden8192_plan_runs_one_group_on_cta_pairs(nest):
                           cta_pairs=False)
     assert q["kernel"] == "tc_wide2_kernel"
     assert (q["groups"], q["parts"], q["stages"]) == (1, SMS, 3)
-    # batches of 129 to 256 queries are one group; more are several
+    # batches of 129 to 512 queries are one group on pairs; more are groups of
+    # 256 on single CTAs
     for B, kernel in ((129, "tc_wide_pair_kernel"), (128, "tc_wide_kernel"),
-                      (257, "tc_wide2_kernel")):
+                      (257, "tc_wide_pair_kernel"), (513, "tc_wide2_kernel")):
         assert nest.plan_offline(1 << 23, 8192, "bf16", B, 1024, num_sms=SMS,
                                  smem_per_block=SMEM)["kernel"] == kernel, B
 
@@ -122,8 +128,10 @@ def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
             assert p["scratch_bytes"] >= groups * p["parts"] * qpg * r * 8, tag
         else:
             assert not c["ragged"] and c["dtype"] == "bf16", tag
-            # pairs when forced, or automatically for a single group of 256
-            assert (p["path"] == 4) == (qpg == 256 and (pairs_of(c) or groups == 1)), tag
+            # pairs when forced, or automatically for one group of up to 512
+            assert (p["path"] == 4) == (qpg >= 256 and (pairs_of(c) is True or B <= 512)), tag
+            # groups of 512 only on pairs, and only for 257 to 512 queries
+            assert (qpg == 512) == (p["path"] == 4 and 256 < B <= 512), tag
             if p["single_pass"]:
                 assert p["sample_stride"] == 1 and p["list_capacity"] == N, tag
             else:
@@ -164,6 +172,9 @@ def test_largest_tensor_core_datastore_keeps_32_bit_lists(nest):
     N = 0x7FFFFF00
     for B, r in [(17, 1), (64, 1024), (512, 4096)]:
         p = nest.plan_offline(N, 8, "bf16", B, r, num_sms=SMS, smem_per_block=SMEM)
-        assert p["path"] in (2, 3), p
+        assert p["path"] in (2, 3, 4), p
         assert p["list_capacity"] < 2 ** 31, p
-        assert p["list_capacity"] <= N // 8 + p["parts"] * 8 * 1024, p
+        # each part has up to 8 reserving warps per column (16 on a pair with
+        # two 256-key tiles per step), each holding a block of at most 1024 slots
+        warps = 16 if p["path"] == 4 else 8
+        assert p["list_capacity"] <= N // 8 + p["parts"] * warps * 1024, p
