@@ -358,7 +358,10 @@ TRAFFIC = {
     ("hidden8192", "tc_wide_pair_kernel", 256): 9239347456 * 8388608 / 557056 + 79070208,
     # tc_wide2_kernel main pass, same workload on single CTAs (--cta-pairs off)
     ("hidden8192", "tc_wide2_kernel", 256): 9177019648 * 8388608 / 557056 + 35045632,
-    # tc_wide2_kernel main pass, large batch: a 262,144-key capture; reads x16, writes as they are
+    # tc_wide_pair_kernel<1> main pass, large batch (one group of 512 on CTA pairs, the
+    # default): a 262,144-key capture; reads x16, writes (mostly reservation padding) as they are
+    ("large_batch", "tc_wide_pair_kernel", 512): 2237294848 * 16 + 38704128,
+    # tc_wide2_kernel main pass, large batch on single CTAs (--cta-pairs off): same capture size
     ("large_batch", "tc_wide2_kernel", 512): 2363021056 * 16 + 33024256,
     # tc_scan_kernel<4>, decode: a 65,536-key capture; reads x16, per-CTA list writes as they are
     ("decode", "tc_scan_kernel", 4): 537274880 * 16 + 2926080,
