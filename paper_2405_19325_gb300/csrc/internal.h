@@ -199,6 +199,7 @@ struct GselectArgs {
     uint32_t* refine_state;  // with words_out: the exact re-ranking's state, reset per query
     unsigned long long* refine_apair;
     int* status;          // with words_out: NEST_ERR_OVERFLOW if a list is still over capacity
+                          // (or held repeated words, which the scans never write)
     // Recovery preparation (instead of any output): for an overflowed list,
     // lim_out[q] = the r-th smallest word it holds; for a list with fewer
     // than r real words (when check_underflow), lim_out[q] = every word up to

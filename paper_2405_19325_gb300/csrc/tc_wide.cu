@@ -1183,8 +1183,17 @@ __global__ void __launch_bounds__(kSelThreads, 1) gselect_kernel(const GselectAr
         select_smallest<kSelThreads, 1>(list, 0, &sh.cnt, &sh.thr, a.r, sh.sel, tid,
                                         [] { __syncthreads(); });
         nsel = sh.cnt;
-        for (int j = tid; j < nsel; j += kSelThreads) stage[j] = list[j];
     }
+    // The select leaves at most r words because the words of a list are
+    // distinct (each carries its key index).  More would mean a list held
+    // repeated words: recorded, and no more than r are used, so that nothing
+    // is written past the r words the stage and the outputs hold.
+    if (nsel > a.r) {
+        if (tid == 0 && a.status != nullptr) record_status(a.status, NEST_ERR_OVERFLOW);
+        nsel = a.r;
+    }
+    if (m < 0)
+        for (int j = tid; j < nsel; j += kSelThreads) stage[j] = list[j];
     if (a.lim_out != nullptr) {
         // Recovery preparation of an overflowed list: the r-th smallest of
         // the words it holds bounds the r-th smallest of all keys from
