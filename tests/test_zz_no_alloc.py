@@ -9,8 +9,8 @@ ABI:
 
 * its results against nest_knn_search on the same inputs, for two calls in
   a row (the shared array keeps the first call's contents), on the narrow
-  scan, the ragged scan and the large-batch path, each right after a call of
-  another shape;
+  scan, the ragged scan, the large-batch path and its CTA-pair kernels, each
+  right after a call of another shape;
 * one case against the fp64 oracle directly;
 * that a call on a fresh handle takes no device memory (the free memory the
   driver reports does not change), while nest_knn_search on another fresh
@@ -124,6 +124,22 @@ def test_static_search_large_batch_path_after_another_shape(nest):
     for seed in (41, 42):
         _static_then_reference(nest, lib, ds, _queries(seed, K, 32), 16)
     ds.close()
+
+
+def test_static_search_on_cta_pairs(nest):
+    """Batches of 129 to 512 queries run on CTA pairs (clusters of two CTAs)
+    by default; through the static entry point too, as one group of 256
+    (B = 200) and as one group of 512 (B = 300), each twice in a row after a
+    narrow search of another shape."""
+    lib = nest.load_library()
+    for B, N in ((200, 4000), (300, 2500)):
+        K, V = _inputs(7 + B, N=N, d=128, centres=10)
+        ds = nest.Datastore(K, V, 1000)
+        assert ds.search_path(B, 16) == "tc_wide_pair_kernel"
+        _static_then_reference(nest, lib, ds, _queries(70 + B, K, 2), 300)
+        for seed in (71 + B, 72 + B):
+            _static_then_reference(nest, lib, ds, _queries(seed, K, B), 16)
+        ds.close()
 
 
 def test_static_search_matches_the_oracle(nest):
