@@ -21,13 +21,19 @@
 //                       at once (8 or 16 KiB rows), and rewrites the word in
 //                       place; each CTA folds its screening errors into the
 //                       query's state with atomics.
+//   then, for a few queries (B < kSortMinB):
 //   refine_rank_kernel  grid (chunks of 16 candidates, B queries), 512
 //                       threads: warp w of chunk c takes candidate 16 c + w,
 //                       counts the query's words below its own (the words
 //                       are distinct, so the counts are the sorted
 //                       positions), and writes s and idx at that position
 //                       when it is below r.  No sort and no CTA that waits
-//                       for the others.
+//                       for the others: r' x r' comparisons per query spread
+//                       over r' / 16 CTAs, which suits a handful of queries;
+//   or, for more queries:
+//   refine_sort_kernel  one 1024-thread CTA per query sorts its r' words in
+//                       shared memory (bitonic network, O(r' log^2 r')
+//                       compare-exchanges) and writes the first r.
 //
 // It also checks the margin.  A key left out of the r' candidates had a
 // screened distance of at least A, the largest screened distance kept.  The
@@ -47,6 +53,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "select.cuh"
 
 namespace nest {
 namespace {
@@ -55,6 +62,13 @@ constexpr int kRefineThreads = 512;
 constexpr int kRefineRows = kRefineThreads / 32;  // candidates per CTA
 constexpr int kRefineLoads = 16;                  // 16-byte loads in flight per lane
 constexpr int kRankThreads = 512;  // one warp per position, 16 per CTA
+constexpr int kSortThreads = 1024;
+// From this many queries on, each query's words are sorted by one CTA
+// instead of ranked by r' / 16 CTAs.  One CTA sorts r' = 1,088 words in
+// about 20 us; the rank kernel spends about 0.38 us per query at that r'
+// once its grid fills the GPU (97 against 29 us at B = 256 on a GB300, about
+// even at B = 64, and the rank kernel ahead below).
+constexpr int kSortMinB = 96;
 // Distance bits no real distance has (a NaN pattern above +inf's bits).
 constexpr uint64_t kPadHigh = 0xFFFFFFFFull << 32;
 
@@ -165,6 +179,20 @@ __global__ void __launch_bounds__(kRefineThreads) refine_dist_kernel(const Refin
     }
 }
 
+// The margin of query b, given its r-th smallest exact word.  Keys outside
+// the candidates exist only when the list is full (the callers check n ==
+// rp); the kernel that writes the lists resets the state.
+__device__ __forceinline__ void check_margin(const RefineArgs& a, int b, uint64_t rth)
+{
+    const float A_exact = __uint_as_float((uint32_t)a.apair[b]);
+    const float emax = from_ordered_bits(a.state[b]);
+    const float emin = from_ordered_bits(a.state[a.B + b]);
+    const float Dr = __uint_as_float((uint32_t)(rth >> 32));
+    const float W = 2.f * (emax - emin);
+    const bool ok = (A_exact - W > Dr) || (A_exact == Dr);
+    if (!ok) record_status(a.status, NEST_ERR_MARGIN);
+}
+
 __global__ void __launch_bounds__(kRankThreads) refine_rank_kernel(const RefineArgs a)
 {
     extern __shared__ __align__(16) uint64_t words[];  // the query's n words
@@ -199,20 +227,44 @@ __global__ void __launch_bounds__(kRankThreads) refine_rank_kernel(const RefineA
                 io[rank] = -1;
             }
         }
-        if (lane == 0 && rank == a.r - 1 && n == a.rp) {
-            // The margin (keys outside the candidates exist only when the
-            // list is full); the kernel that writes the lists resets the state.
-            const float A_exact = __uint_as_float((uint32_t)a.apair[b]);
-            const float emax = from_ordered_bits(a.state[b]);
-            const float emin = from_ordered_bits(a.state[a.B + b]);
-            const float Dr = __uint_as_float((uint32_t)(mine >> 32));
-            const float W = 2.f * (emax - emin);
-            const bool ok = (A_exact - W > Dr) || (A_exact == Dr);
-            if (!ok) record_status(a.status, NEST_ERR_MARGIN);
-        }
+        if (lane == 0 && rank == a.r - 1 && n == a.rp) check_margin(a, b, mine);
     } else if (i < a.r && lane == 0) {
         so[i] = -INFINITY;  // positions n .. r - 1 of a short row
         io[i] = -1;
+    }
+}
+
+// One CTA per query: its n words (exact distances : key), padded to P2 (a
+// power of two >= max(r', r)) with distinct words above every real one,
+// sorted ascending; position j < r gives s and idx, as refine_rank_kernel
+// writes them.
+__global__ void __launch_bounds__(kSortThreads) refine_sort_kernel(const RefineArgs a, int P2)
+{
+    extern __shared__ __align__(16) uint64_t sorted[];  // P2 words
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int tid = threadIdx.x;
+    const int b = blockIdx.x;
+    const uint64_t* list = a.cand + (int64_t)b * a.rp;
+    const int n = min(max(a.cand_cnt[b], 0), a.rp);
+    for (int i = tid; i < P2; i += kSortThreads) {
+        const uint64_t w = i < n ? list[i] : kNoCandidate;
+        sorted[i] = w != kNoCandidate ? w : (kPadHigh | (uint32_t)i);
+    }
+    __syncthreads();
+    bitonic_sort<kSortThreads>(sorted, P2, tid, [] { __syncthreads(); });
+    float* so = a.s_out + (int64_t)b * a.r;
+    int64_t* io = a.idx_out + (int64_t)b * a.r;
+    for (int j = tid; j < a.r; j += kSortThreads) {
+        const uint64_t w = sorted[j];
+        if ((w >> 32) < 0xFFFFFFFFu) {
+            so[j] = -__uint_as_float((uint32_t)(w >> 32));
+            io[j] = (int64_t)(uint32_t)w;
+        } else {
+            so[j] = -INFINITY;
+            io[j] = -1;
+        }
+        if (j == a.r - 1 && n == a.rp) check_margin(a, b, w);
     }
 }
 
@@ -246,8 +298,16 @@ cudaError_t launch_refine(int dtype, const RefineArgs& a, cudaStream_t stream)
             e = launch_pdl(refine_dist_kernel<NEST_F32>, grid, dim3(kRefineThreads), qbytes, stream, a);
     }
     if (e != cudaSuccess) return e;
-    // rank threads cover max(r', r) positions: candidates, then the padding of short rows
     const int cover = a.rp > a.r ? a.rp : a.r;
+    if (a.B >= kSortMinB) {
+        int P2 = 1;
+        while (P2 < cover) P2 <<= 1;
+        const size_t sbytes = (size_t)P2 * sizeof(uint64_t);
+        e = raise_smem_limit(reinterpret_cast<const void*>(refine_sort_kernel), sbytes);
+        if (e != cudaSuccess) return e;
+        return launch_pdl(refine_sort_kernel, dim3(a.B), dim3(kSortThreads), sbytes, stream, a, P2);
+    }
+    // rank threads cover max(r', r) positions: candidates, then the padding of short rows
     const dim3 rgrid((cover + kRankThreads / 32 - 1) / (kRankThreads / 32), a.B);
     const size_t wbytes = (size_t)a.rp * sizeof(uint64_t);
     e = raise_smem_limit(reinterpret_cast<const void*>(refine_rank_kernel), wbytes);
