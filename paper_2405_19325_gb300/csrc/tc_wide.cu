@@ -1,27 +1,35 @@
 // tc_wide.cu -- the search for large query batches (Sec. 2.2 / App. A: the
 // r nearest keys of each query, s = -||q - k||^2), where per-query candidate
-// lists no longer fit in one CTA's shared memory.
+// lists no longer fit in one CTA's shared memory.  "r" below is the number
+// of screened candidates the search keeps for the exact re-ranking
+// (refine.cu), r' = r + margin of the caller.
 //
 //   0. wide_qnorm_kernel computes ||q||^2 of every query once.
 //   1. A sampling pre-pass: the scan kernel over a tensor map that reads
 //      every stride-th key, admitting every sampled key (each list holds the
-//      sample in row order), and gselect_kernel on those lists give each
-//      query the r-th distance among the sample.  It is an upper bound of the
-//      query's true r-th distance, so every key at or below it is a safe
-//      candidate (admission threshold).
-//   2. The main pass streams every key tile once per group of up to 256
-//      queries with tcgen05.mma (M = 128 keys, N = up to 256 queries,
-//      K = 16): tc_wide_kernel keeps one key tile per stage and two TMEM
-//      accumulators of N columns.  Groups of 256 run on tc_wide2_kernel
-//      (two key tiles per stage, one accumulator each) or on CTA pairs
-//      (tc_wide_pair_kernel: M = 256 keys over the pair; the default when
-//      the batch is one group of up to 512 queries).  The epilogue warps form
-//      ||q||^2 + ||k||^2 - 2 q.k, admit the keys under each query's threshold
-//      and append them to that query's global list through per-warp slot
-//      reservations.
-//   3. gselect_kernel takes the exact r smallest of each list (three
-//      streaming passes, then a select in shared memory), sorts them and
-//      writes s and idx.
+//      sample in row order), then gselect_kernel sorts each query's r
+//      nearest sampled keys.  The sample's r-th distance bounds the query's
+//      true r-th distance from above.
+//   2. The main pass streams every key once per group of queries with
+//      tcgen05.mma (M = 128 keys, N = up to 256 queries, K = 16):
+//      tc_wide_kernel keeps one key tile per stage and two TMEM accumulators
+//      of N columns; groups of 256 run on tc_wide2_kernel (two key tiles per
+//      stage, one accumulator each) or on CTA pairs (tc_wide_pair_kernel:
+//      M = 256 keys over the pair, groups of 256 or 512; the default when the
+//      batch is one group).  The epilogue warps form ||q||^2 + ||k||^2 -
+//      2 q.k, admit the keys up to the sample's j-th distance (an optimistic
+//      threshold, j = max(32, 4 r / stride), that lets about 4 r keys
+//      through) and append them to that query's global list through
+//      per-warp slot reservations.
+//   3. Recovery, up to three rounds of two kernels that return at once when
+//      nothing needs them: gselect_kernel in preparation mode flags a list
+//      with fewer than r real words (scanned again up to the sample's r-th
+//      distance) or one that overflowed its capacity (scanned again up to
+//      the r-th smallest word it holds), and tc_wide_kernel<NM, true>
+//      rescans the flagged groups.
+//   4. gselect_kernel takes the exact r smallest words of each list (three
+//      streaming passes, then a select in shared memory) for the exact
+//      re-ranking.
 #include <cmath>
 #include <cuda.h>
 
