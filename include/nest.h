@@ -385,7 +385,8 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
 
 /*
  * Which distance scan a search of this shape runs on this datastore:
- *   0  CUDA-core scan with per-CTA top-r (fp32 keys, or rows TMA cannot map)
+ *   0  CUDA-core scan with per-CTA top-r (fp32 keys with rows over 2 KiB,
+ *      or rows TMA cannot map)
  *   1  tensor-core scan with per-CTA top-r (bf16 keys, query groups of <= 16)
  *   2  tensor-core scan of large query batches against sampled admission
  *      thresholds (bf16 keys, more queries than one CTA keeps lists for)
@@ -394,6 +395,8 @@ NEST_API nest_status_t nest_timing_read(nest_datastore_t* ds, double* total_ms, 
  *   4  the same on CTA pairs (groups of 256 or 512 queries, 256-key tiles
  *      split over two SMs): by default for 129 to 512 queries; see
  *      nest_datastore_use_cta_pairs
+ *   5  CUDA-core scan of fp32 keys with rows of at most 2 KiB (d <= 512), one
+ *      key row per thread, with per-CTA top-r
  * Returns a negative nest_status_t on a bad argument.  Host only, no launch.
  */
 NEST_API int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r,
@@ -415,7 +418,7 @@ typedef struct nest_plan {
     int32_t queries_per_group;  /* queries one CTA (or CTA pair) scans together */
     int32_t groups;             /* query groups */
     int32_t parts;              /* key-range parts per group (CTAs or CTA pairs) */
-    int32_t stages;             /* pipeline stages of the scan kernel */
+    int32_t stages;             /* pipeline stages of the scan kernel (1 for path 5) */
     int32_t single_pass;        /* paths 2-4: 1 when the sample is every key */
     int64_t sample_stride;      /* paths 2-4: the sample is every stride-th key */
     int64_t list_capacity;      /* words of a query's candidate list: in a CTA's shared
@@ -439,7 +442,7 @@ NEST_API const char* nest_status_string(nest_status_t status);
 /* ABI version: major * 10000 + minor * 100 + patch (0.2.0: CTA pairs and
  * the bounded-wait self-test added to 0.1.0; 0.3.0: CTA pairs with 48 KiB
  * stages and groups of up to 512 queries, chosen automatically for one
- * query group). */
+ * query group; search path 5 for narrow fp32 rows). */
 NEST_API int32_t nest_version(void);
 
 #ifdef __cplusplus

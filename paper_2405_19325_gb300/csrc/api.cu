@@ -72,6 +72,7 @@ struct SearchPlan {
     int r;         // neighbours returned
     int rp;        // screened candidates kept per query for the exact re-ranking
     bool tc;       // tensor-core scan (bf16) or CUDA-core scan
+    bool rows;     // CUDA-core scan of narrow fp32 rows, one row per thread (scan_rows.cu)
     ScanPlan scan;
     TcPlan tcp;
     int nq, groups, parts;
@@ -159,7 +160,28 @@ nest_status_t plan_search(const nest_datastore* ds, int B, int r_out, bool ragge
             sp->parts = tp.parts;
         }
     }
-    if (!sp->tc) {
+    sp->rows = false;
+    if (!sp->tc && ds->dtype == NEST_F32 && ds->row_bytes <= kRowsMaxBytes) {
+        // narrow fp32 rows: one row per thread (scan_rows.cu), several CTAs per SM
+        int nq = ragged ? 1 : ceil_pow2(std::min(B, 8));
+        ScanPlan p{};
+        while (!rows_plan_smem(nq, r, ds->row_bytes, ds->smem_optin, &p)) {
+            if (nq == 1) return NEST_ERR_UNSUPPORTED;
+            nq /= 2;
+        }
+        p.groups = ragged ? B : (B + nq - 1) / nq;
+        const int64_t keys_per_group = ragged ? (ds->N + B - 1) / B : keys_per_group_full;
+        // up to four CTAs per SM (the kernel's register budget) count as
+        // slots: more parts would only add lists to merge
+        const int slots = ds->num_sms * std::min(p.ctas_per_sm, kRowsCtasPerSm);
+        p.parts = choose_parts(p.groups, keys_per_group, slots, ragged);
+        sp->rows = true;
+        sp->scan = p;
+        sp->nq = p.nq;
+        sp->groups = p.groups;
+        sp->parts = p.parts;
+    }
+    if (!sp->tc && !sp->rows) {
         const int chunks = ds->row_bytes / 16;
         const int cpt = chunks <= 256 ? 1 : (chunks <= 512 ? 2 : 4);
         int nq = ragged ? 1 : (B >= 3 ? 4 : B);
@@ -688,7 +710,8 @@ nest_status_t launch_search(nest_datastore* ds, const void* q, int32_t B, int32_
             sa.stages = sp.scan.stages;
             sa.stage_bytes = sp.scan.stage_bytes;
             if (timed && (st = record_event(ds, stream)) != NEST_OK) return st;
-            e = launch_scan(ds->dtype, sp.scan, sa, stream);
+            e = sp.rows ? launch_scan_rows(sp.scan, sa, stream)
+                        : launch_scan(ds->dtype, sp.scan, sa, stream);
         }
         if (e != cudaSuccess) return from_cuda(e);
         ++ds->launches;
@@ -1201,7 +1224,7 @@ nest_status_t nest_plan_offline(int64_t N, int32_t d, nest_dtype_t dtype, int32_
     const nest_status_t st = plan_search(&ds, B, r, ragged != 0, &sp);
     if (st != NEST_OK) return st;
     nest_plan_t p{};
-    p.path = sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : 0);
+    p.path = sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : (sp.rows ? 5 : 0));
     if (sp.wide) {
         p.queries_per_group = sp.wpm.nm;
         p.groups = sp.wpm.groups;
@@ -1228,7 +1251,7 @@ int32_t nest_search_path(const nest_datastore_t* ds, int32_t B, int32_t r, int32
     SearchPlan sp;
     const nest_status_t st = plan_search(ds, B, r, ragged != 0, &sp);
     if (st != NEST_OK) return -(int32_t)st;
-    return sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : 0);
+    return sp.wide ? (sp.wpm.pair ? 4 : (sp.wpm.mb == 2 ? 3 : 2)) : (sp.tc ? 1 : (sp.rows ? 5 : 0));
 }
 
 const char* nest_status_string(nest_status_t s)

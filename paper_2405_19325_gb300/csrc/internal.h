@@ -72,6 +72,7 @@ struct ScanPlan {
     int stages;       // pipeline depth
     int stage_bytes;  // bytes of one stage (kScanRows rows)
     size_t smem;      // dynamic shared memory of one CTA
+    int ctas_per_sm;  // scan_rows.cu: CTAs one SM holds at once
 };
 
 constexpr int kScanRows = 4;           // key rows per pipeline stage
@@ -100,6 +101,17 @@ struct ScanArgs {
 // Returns false if no kernel exists for (dtype, nq, cpt).
 bool scan_plan_smem(int dtype, int nq, int cpt, int r, int row_bytes, size_t smem_limit,
                     ScanPlan* plan);
+
+// ---------------------------------------------------------------- scan_rows.cu
+// fp32 keys with rows of at most kRowsMaxBytes: one key row per thread of a
+// 128-thread CTA, NQ = 1, 2, 4 or 8 queries per CTA (ScanPlan: nq, cap,
+// smem, ctas_per_sm; groups and parts set by the caller).  Same arguments
+// and outputs as the scan above.
+constexpr int kRowsThreads = 128;
+constexpr int kRowsCtasPerSm = 4;  // the kernels' register budget: 128 per thread
+constexpr int kRowsMaxBytes = 2048;
+bool rows_plan_smem(int nq, int r, int row_bytes, size_t smem_limit, ScanPlan* plan);
+cudaError_t launch_scan_rows(const ScanPlan& plan, const ScanArgs& args, cudaStream_t stream);
 cudaError_t launch_scan(int dtype, const ScanPlan& plan, const ScanArgs& args,
                         cudaStream_t stream);
 

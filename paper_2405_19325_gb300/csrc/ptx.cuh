@@ -285,6 +285,27 @@ __device__ __forceinline__ void st_shared_u32_if(bool pred, const uint32_t* p, u
         "r"(smem_addr(p)), "r"(v));
 }
 
+// ---------------------------------------------------------------- per-thread async copies
+// 16 bytes from global to shared memory without passing through registers
+// (L2 only); src_bytes = 0 writes zeros and reads nothing.  Both addresses
+// are 16-byte aligned.
+__device__ __forceinline__ void cp_async_16(void* dst_smem, const void* src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst_smem)),
+                 "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit()
+{
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// Waits until at most N of this thread's committed groups are still in flight.
+template <int N>
+__device__ __forceinline__ void cp_async_wait()
+{
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // ---------------------------------------------------------------- CTA pairs (cluster of 2)
 // A pair's tcgen05 work (M = 256 split over both CTAs' shared memory and
 // TMEM) is issued by the even CTA; the odd CTA's operand halves sit at the

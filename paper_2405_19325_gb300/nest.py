@@ -408,7 +408,7 @@ class Datastore:
         return int(self._lib.nest_launch_count(self._h))
 
     SEARCH_PATHS = {0: "scan_topr_kernel", 1: "tc_scan_kernel", 2: "tc_wide_kernel",
-                    3: "tc_wide2_kernel", 4: "tc_wide_pair_kernel"}
+                    3: "tc_wide2_kernel", 4: "tc_wide_pair_kernel", 5: "scan_rows_kernel"}
 
     def search_path(self, B: int, r: int, ragged: bool = False) -> str:
         """Name of the distance-scan kernel a search of this shape runs."""

@@ -100,7 +100,7 @@ def test_verify_spans_matches_oracle(nest):
 
 @pytest.mark.parametrize("path,B,r,dtype,N", [("tc_scan_kernel", 4, 64, "bf16", 60000),
                                                ("tc_wide_kernel", 40, 128, "bf16", 60000),
-                                               ("scan_topr_kernel", 3, 50, "f32", 60000),
+                                               ("scan_rows_kernel", 3, 50, "f32", 60000),
                                                # groups of 256: one pass, then two passes,
                                                # on CTA pairs and on single CTAs
                                                ("tc_wide_pair_kernel", 300, 128, "bf16", 60000),

@@ -279,7 +279,7 @@ def test_sweep_reaches_every_search_path(nest):
                                      cta_pairs=_pairs(c))
             assert plan["kernel"] == path, (c, plan)
     assert seen >= {"tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
-                    "tc_wide_pair_kernel", "scan_topr_kernel"}, seen
+                    "tc_wide_pair_kernel", "scan_topr_kernel", "scan_rows_kernel"}, seen
 
 
 # ---------------------------------------------------------------- Eq. 7 verification and masking

@@ -90,8 +90,16 @@ def test_ragged_and_fp32_plans(nest):
                           smem_per_block=SMEM)
     assert p["kernel"] == "tc_scan_kernel"
     assert (p["queries_per_group"], p["groups"]) == (1, 32)  # one query per CTA, own segment
+    # fp32 keys: narrow rows one per thread (the tiny workload: 256-byte rows,
+    # all 8 queries in one CTA), wide rows on the column-chunk scan
     p = nest.plan_offline(4096, 64, "f32", 8, 16, num_sms=SMS, smem_per_block=SMEM)
-    assert p["kernel"] == "scan_topr_kernel"
+    assert p["kernel"] == "scan_rows_kernel"
+    assert (p["queries_per_group"], p["groups"], p["stages"]) == (8, 1, 1)
+    assert p["list_capacity"] >= (16 + 16) + 128  # r' plus a tile of appends
+    assert nest.plan_offline(1 << 20, 512, "f32", 8, 16, num_sms=SMS,
+                             smem_per_block=SMEM)["kernel"] == "scan_rows_kernel"
+    assert nest.plan_offline(1 << 20, 516, "f32", 8, 16, num_sms=SMS,
+                             smem_per_block=SMEM)["kernel"] == "scan_topr_kernel"
 
 
 def test_large_batch_single_pass_when_the_sample_is_every_key(nest):
@@ -116,13 +124,14 @@ def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
         tag = f"{c}: {p}"
         qpg, groups = p["queries_per_group"], p["groups"]
         # the smallest ring each kernel is planned with
-        assert p["parts"] >= 1 and p["stages"] >= {0: 2, 1: 4, 2: 3, 3: 3, 4: 4}[p["path"]], tag
-        assert (c["dtype"] == "f32") == (p["path"] == 0), tag
+        assert p["parts"] >= 1 and p["stages"] >= {0: 2, 1: 4, 2: 3, 3: 3, 4: 4, 5: 1}[p["path"]], tag
+        assert (c["dtype"] == "f32") == (p["path"] in (0, 5)), tag
+        assert (p["path"] == 5) == (c["dtype"] == "f32" and d * 4 <= 2048), tag
         if c["ragged"]:
             assert qpg == 1 and groups == B, tag
         else:
             assert groups * qpg >= B > (groups - 1) * qpg, tag
-        if p["path"] <= 1:
+        if p["path"] in (0, 1, 5):
             # room for a list of r plus the appends of at least one block of keys
             assert p["list_capacity"] > r, tag
             assert p["scratch_bytes"] >= groups * p["parts"] * qpg * r * 8, tag
@@ -142,7 +151,8 @@ def test_plans_of_every_sweep_shape_keep_the_invariants(nest):
                 assert N // p["sample_stride"] >= target, tag
                 assert p["list_capacity"] >= min(N, 8 * rp), tag
             assert p["scratch_bytes"] >= B * p["list_capacity"] * 8, tag
-    assert seen >= {"scan_topr_kernel", "tc_scan_kernel", "tc_wide_kernel", "tc_wide2_kernel",
+    assert seen >= {"scan_topr_kernel", "scan_rows_kernel", "tc_scan_kernel", "tc_wide_kernel",
+                    "tc_wide2_kernel",
                     "tc_wide_pair_kernel"}, seen
 
 
