@@ -702,14 +702,16 @@ def test_large_batch_full_size_sampled_rows(nest):
 def test_hidden8192_full_size_B_sweep(nest):
     """bf16 d=8192, N=8,388,608 clustered keys (128 GiB), r=1024, B in {1, 8, 64, 256}:
     four kernel paths on one datastore, each checked against the oracle on the
-    rows it shares with a fixed set of 32 rows (0-7, eight more below 64 and
-    sixteen spread to 255); the oracle scans all keys once for those rows."""
+    rows it shares with a fixed set of 48 rows (0-7, 24 more spread below 64
+    and 16 spread to 255), so that B = 64 and B = 256 are checked on at least
+    32 rows and B = 1 and 8 on all of theirs; the oracle scans all keys once
+    for those rows."""
     w = synth.WORKLOADS["hidden8192"]
     x = synth.make_inputs(w, device="cuda", B=256)
     ds = nest.Datastore(x.K, x.V, w.vocab)
-    rows = sorted(set(range(8)) | {9, 17, 25, 33, 41, 49, 57, 63}
+    rows = sorted(set(range(8)) | set(np.linspace(8, 63, 24).round().astype(int).tolist())
                   | set(np.linspace(64, 255, 16).round().astype(int).tolist()))
-    assert len(rows) == 32
+    assert len(rows) == 48 and sum(b < 64 for b in rows) == 32
     q_np = synth.to_numpy_raw(x.q[rows])
     s_or, i_or = _oracle_rows_parallel(x.K, q_np, w.r)
     for B in (1, 8, 64, 256):
