@@ -316,7 +316,6 @@ struct RefineArgs {
 };
 
 int refine_margin(int r);
-size_t refine_smem_bytes(int rp, int r, int row_bytes);
 cudaError_t launch_refine(int dtype, const RefineArgs& args, cudaStream_t stream);
 
 // ---------------------------------------------------------------- mix.cu

@@ -276,13 +276,6 @@ int refine_margin(int r)
     return m < 16 ? 16 : (m > 128 ? 128 : m);
 }
 
-size_t refine_smem_bytes(int rp, int r, int row_bytes)
-{
-    (void)r;
-    const size_t words = (size_t)rp * sizeof(uint64_t);
-    return words > (size_t)row_bytes ? words : (size_t)row_bytes;
-}
-
 cudaError_t launch_refine(int dtype, const RefineArgs& a, cudaStream_t stream)
 {
     const dim3 grid((a.rp + kRefineRows - 1) / kRefineRows, a.B);
