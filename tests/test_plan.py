@@ -100,6 +100,12 @@ def test_ragged_and_fp32_plans(nest):
                              smem_per_block=SMEM)["kernel"] == "scan_rows_kernel"
     assert nest.plan_offline(1 << 20, 516, "f32", 8, 16, num_sms=SMS,
                              smem_per_block=SMEM)["kernel"] == "scan_topr_kernel"
+    # ragged fp32 segments: one query per CTA group on either fp32 scan
+    for d, kernel in ((64, "scan_rows_kernel"), (1024, "scan_topr_kernel")):
+        p = nest.plan_offline(32 * 2560, d, "f32", 32, 16, ragged=True, num_sms=SMS,
+                              smem_per_block=SMEM)
+        assert p["kernel"] == kernel
+        assert (p["queries_per_group"], p["groups"]) == (1, 32)
 
 
 def test_large_batch_single_pass_when_the_sample_is_every_key(nest):
