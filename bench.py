@@ -659,6 +659,9 @@ def measure(args, w, x_all, ds, B, world, rank, local, light=False):
         d2h = res_h.numel() * res_h.element_size()
     # about three seconds of end-to-end steps at most (and at least five)
     n_e2e = max(5, min(args.e2e_steps, int(3000.0 / max(step_ms, 1e-3))))
+    # clocks of this loop too: it runs seconds after the timed region, and
+    # where the power cap sets the clock the two can differ by a few per cent
+    e2e_clocks = Clocks(local)
     for _ in range(3):
         e2e_step()
     barrier(world)
@@ -668,7 +671,8 @@ def measure(args, w, x_all, ds, B, world, rank, local, light=False):
     e2e_s = max_over_ranks(time.perf_counter() - te, world)
     e2e = {"value": world * B * n_e2e / e2e_s,
            "unit": "positions/s" if args.pipeline == "verify" else "queries/s",
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e}
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
+           "clocks": e2e_clocks.stop()}
 
     unit = "positions/s" if args.pipeline == "verify" else "queries/s"
     if light:
